@@ -1,0 +1,184 @@
+"""CPU oracle for CacheBack's score -> select -> compact path (fp64).
+
+TEST INFRASTRUCTURE, NOT PRODUCT CODE.  Only `tests/`, `__graft_entry__.smoke()`
+and the CPU-baseline / reference leg of `bench.py` may import this package.
+It shares nothing with the CUDA path: the arithmetic lives in `cb_oracle.c`
+(plain C, fp64, OpenMP over KV-head groups with a fixed-order final sum), built
+here with gcc; `brute.py` is a second, literal numpy restatement used only on
+tiny inputs.
+
+Functions (each follows the paper's App. C.1 / C.2 in its own order):
+  score(K, Q, ...)        -> dict of fp64 [T] arrays: S, Q, C, U, N, D
+  attention(K, Q, scale)  -> a[l][h][r][t]
+  select(S, B, ...)       -> int32 indices, ascending
+  compact(K, V, idx, ...) -> gathered K, V rows
+  budget(T, keep)         -> ceil(keep * T) in double, clamped to [0, T]
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import subprocess
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "cb_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "libcb_oracle.so")
+CFLAGS = ["-O2", "-ffp-contract=off", "-fopenmp", "-fPIC", "-shared", "-Wall", "-Wextra"]
+
+OK, EINVAL, ESHAPE, EBUDGET, ENOMEM = 0, 1, 2, 3, 4
+
+
+def build(src: str = _SRC, out: str = _LIB_PATH, force: bool = False) -> str:
+    """Compile the oracle with gcc (no nvcc, no CUDA)."""
+    if not force and os.path.exists(out) and os.path.getmtime(out) >= os.path.getmtime(src):
+        return out
+    tmp = out + ".tmp%d" % os.getpid()
+    subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, src, "-lm"])
+    os.replace(tmp, out)
+    return out
+
+
+class _Dims(ctypes.Structure):
+    _fields_ = [
+        ("n_layers", ctypes.c_int32), ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32), ("m", ctypes.c_int32), ("T", ctypes.c_int64),
+        ("k_layer", ctypes.c_int64), ("k_head", ctypes.c_int64), ("k_pos", ctypes.c_int64),
+        ("q_layer", ctypes.c_int64), ("q_tok", ctypes.c_int64), ("q_head", ctypes.c_int64),
+    ]
+
+
+_P = ctypes.c_void_p
+
+
+class Oracle:
+    """ctypes view of one build of cb_oracle.c (the default build, or a test's variant)."""
+
+    def __init__(self, path: Optional[str] = None):
+        self.path = path or build()
+        lib = ctypes.CDLL(self.path)
+        lib.cbo_score.argtypes = [ctypes.POINTER(_Dims), _P, _P, ctypes.c_double, ctypes.c_double,
+                                  ctypes.c_double, ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P, _P, _P]
+        lib.cbo_score.restype = ctypes.c_int
+        lib.cbo_attention.argtypes = [ctypes.POINTER(_Dims), _P, _P, ctypes.c_double, _P]
+        lib.cbo_attention.restype = ctypes.c_int
+        for name, ptr_t in (("cbo_select_f64", _P), ("cbo_select_f32", _P)):
+            f = getattr(lib, name)
+            f.argtypes = [ctypes.c_int64, ptr_t, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                          ctypes.c_int32, _P]
+            f.restype = ctypes.c_int64
+        lib.cbo_compact.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_int64, _P, _P,
+                                    ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
+        lib.cbo_compact.restype = ctypes.c_int
+        lib.cbo_pool.argtypes = [_P, _P, ctypes.c_int64, ctypes.c_int32]
+        lib.cbo_pool.restype = None
+        lib.cbo_max_threads.restype = ctypes.c_int
+        self.lib = lib
+
+    # -- helpers -----------------------------------------------------------
+    @staticmethod
+    def _bits(x) -> np.ndarray:
+        """bf16 tensor/array -> contiguous uint16 bit array (host)."""
+        try:
+            import torch
+            if isinstance(x, torch.Tensor):
+                return x.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        except ImportError:  # pragma: no cover
+            pass
+        a = np.ascontiguousarray(x)
+        if a.dtype != np.uint16:
+            raise TypeError("expected bf16 bits as uint16")
+        return a
+
+    @staticmethod
+    def _dims(Kb: np.ndarray, Qb: np.ndarray) -> _Dims:
+        nL, Hkv, T, d = Kb.shape
+        nL2, m, Hq, d2 = Qb.shape
+        if nL2 != nL or d2 != d:
+            raise ValueError("K and Q disagree on layers or head_dim")
+        return _Dims(nL, Hq, Hkv, d, m, T, Hkv * T * d, T * d, d, m * Hq * d, Hq * d, d)
+
+    def max_threads(self) -> int:
+        return int(self.lib.cbo_max_threads())
+
+    # -- App. C.1 ------------------------------------------------------------
+    def score(self, K, Q, p: float = 2.0, alpha: float = 2.0, pool_w: int = 7,
+              scale: Optional[float] = None, n_threads: int = 0) -> dict:
+        Kb, Qb = self._bits(K), self._bits(Q)
+        dm = self._dims(Kb, Qb)
+        T = dm.T
+        if scale is None:
+            scale = 1.0 / math.sqrt(dm.head_dim)
+        out = {k: np.zeros(T, dtype=np.float64) for k in ("S", "Q", "C", "U", "N", "D")}
+        st = self.lib.cbo_score(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data, scale, p, alpha,
+                                pool_w, n_threads, *(out[k].ctypes.data for k in ("S", "Q", "C", "U", "N", "D")))
+        if st != OK:
+            raise RuntimeError("cbo_score failed with status %d" % st)
+        return out
+
+    def attention(self, K, Q, scale: Optional[float] = None) -> np.ndarray:
+        Kb, Qb = self._bits(K), self._bits(Q)
+        dm = self._dims(Kb, Qb)
+        if scale is None:
+            scale = 1.0 / math.sqrt(dm.head_dim)
+        a = np.zeros((dm.n_layers, dm.n_q_heads, dm.m, dm.T), dtype=np.float64)
+        st = self.lib.cbo_attention(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data, scale, a.ctypes.data)
+        if st != OK:
+            raise RuntimeError("cbo_attention failed with status %d" % st)
+        return a
+
+    def pool(self, x, w: int = 7) -> np.ndarray:
+        x = np.ascontiguousarray(x, dtype=np.float64)
+        y = np.empty_like(x)
+        self.lib.cbo_pool(x.ctypes.data, y.ctypes.data, x.shape[0], w)
+        return y
+
+    # -- App. C.2 ------------------------------------------------------------
+    def select(self, S, B: int, n_sink: int = 1, n_latent: int = 40, span_w: int = 16) -> np.ndarray:
+        """Span selection.  fp32 scores are ranked in fp32, fp64 scores in fp64."""
+        S = np.asarray(S)
+        T = S.shape[0]
+        idx = np.zeros(max(B, 1), dtype=np.int32)
+        if S.dtype == np.float32:
+            S = np.ascontiguousarray(S)
+            n = self.lib.cbo_select_f32(T, S.ctypes.data, B, n_sink, n_latent, span_w, idx.ctypes.data)
+        else:
+            S = np.ascontiguousarray(S, dtype=np.float64)
+            n = self.lib.cbo_select_f64(T, S.ctypes.data, B, n_sink, n_latent, span_w, idx.ctypes.data)
+        if n < 0:
+            raise ValueError("cbo_select failed with status %d" % (-n))
+        return idx[:n]
+
+    def compact(self, K, V, idx, out_k=None, out_v=None, offset: int = 0):
+        Kb, Vb = self._bits(K), self._bits(V)
+        nL, Hkv, T, d = Kb.shape
+        idx = np.ascontiguousarray(idx, dtype=np.int32)
+        B = idx.shape[0]
+        if out_k is None:
+            out_k = np.zeros((nL, Hkv, offset + B, d), dtype=np.uint16)
+            out_v = np.zeros_like(out_k)
+        cap = out_k.shape[2]
+        dm = _Dims(nL, Hkv, Hkv, d, 1, T, Hkv * T * d, T * d, d, 0, 0, 0)
+        st = self.lib.cbo_compact(ctypes.byref(dm), Kb.ctypes.data, Vb.ctypes.data, idx.ctypes.data, B,
+                                  out_k.ctypes.data, out_v.ctypes.data, offset, Hkv * cap * d, cap * d)
+        if st != OK:
+            raise RuntimeError("cbo_compact failed with status %d" % st)
+        return out_k, out_v
+
+
+def budget(T: int, keep: float) -> int:
+    """B = ceil(keep * T) in double, clamped to [0, T] (App. C.2: B_i = ceil(T_i / r), keep = 1/r)."""
+    return int(min(T, max(0, math.ceil(keep * T))))
+
+
+_DEFAULT: Optional[Oracle] = None
+
+
+def default() -> Oracle:
+    global _DEFAULT
+    if _DEFAULT is None:
+        _DEFAULT = Oracle()
+    return _DEFAULT

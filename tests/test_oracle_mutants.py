@@ -1,0 +1,89 @@
+"""Planted mistakes in the oracle must each fail at least one pin (no GPU).
+
+Every entry patches one plausible mistake into a copy of oracle/cb_oracle.c (a
+dropped term, a wrong sign, index or exponent, a transposed operand, a wrong
+tie-break), builds it with gcc, and runs the pins of tests/oracle_pins.py on
+it.  A mutant that passes every pin would mean the pins cannot see that
+mistake.  All mutants keep every memory access in bounds for the pins' sizes.
+"""
+import concurrent.futures as cf
+import os
+import tempfile
+
+import pytest
+
+import oracle
+import oracle_pins
+
+MUTANTS = [
+    ("gqa_mapping_in_attention", "load_keys_transposed(dm, K, l, h / G)", "load_keys_transposed(dm, K, l, h % dm->n_kv_heads)"),
+    ("gqa_mapping_in_score", "const int h = g * G + j;", "const int h = j * Hkv + g;"),
+    ("scale_dropped", "z[t] *= scale;", "z[t] *= 1.0;"),
+    ("softmax_sign", "a[t] = exp(z[t] - M);", "a[t] = exp(M - z[t]);"),
+    ("softmax_not_normalised", "for (int64_t t = 0; t < T; ++t) a[t] /= Z;", "(void)Z;"),
+    ("q_operand_transposed", "(int64_t)r * dm->q_tok + (int64_t)h * dm->q_head", "(int64_t)h * dm->q_tok + (int64_t)r * dm->q_head"),
+    ("k_dim_reversed", "bf16_to_double(base[t * dm->k_pos + k])", "bf16_to_double(base[t * dm->k_pos + (d - 1 - k)])"),
+    ("k_position_shifted", "bf16_to_double(base[t * dm->k_pos + k])", "bf16_to_double(base[((t + 1) % T) * dm->k_pos + k])"),
+    ("group_mean_missing_1_over_G", "br[t] += a[t] / G;", "br[t] += a[t];"),
+    ("layer_term_over_kv_heads", "Us[t] += a[t] / ((double)m * Hq);", "Us[t] += a[t] / ((double)m * Hkv);"),
+    ("numerator_unpooled", "cbo_pool(br, pooled, T, pool_w);", "cbo_pool(br, pooled, T, 1);"),
+    ("denominator_unpooled", "cbo_pool(bbar, pooled, T, pool_w);", "cbo_pool(bbar, pooled, T, 1);"),
+    ("numerator_power_fixed_2", "Ns[t] += pow(pooled[t], p) / m;", "Ns[t] += pooled[t] * pooled[t] / m;"),
+    ("denominator_power_dropped", "Ds[t] = pow(pooled[t], p);", "Ds[t] = pooled[t];"),
+    ("numerator_sum_not_mean", "Ns[t] += pow(pooled[t], p) / m;", "Ns[t] += pow(pooled[t], p);"),
+    ("mean_query_attention_unpooled", "cbo_pool(Usum, Qv, T, pool_w);", "cbo_pool(Usum, Qv, T, 1);"),
+    ("correction_exponent", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))", "pow(Nsum[t] / Dsum[t], 1.0 / p)"),
+    ("correction_ratio_inverted", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))", "pow(Dsum[t] / Nsum[t], 1.0 / (p - 1.0))"),
+    ("strength_exponent_dropped", "if (S) S[t] = Qv[t] * pow(c, alpha);", "if (S) S[t] = Qv[t] * c;"),
+    ("zero_denominator_gives_0", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0)) : 1.0;", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0)) : 0.0;"),
+    ("pool_window_too_wide", "int64_t half = w / 2;", "int64_t half = w / 2 + 1;"),
+    ("pool_window_shifted", "int64_t hi = t + half > T - 1 ? T - 1 : t + half;", "int64_t hi = t + half + 1 > T - 1 ? T - 1 : t + half + 1;"),
+    ("pool_min_not_max", "if (x[u] > mx) mx = x[u];", "if (x[u] < mx) mx = x[u];"),
+    ("span_tie_favours_later", "return a->j < b->j ? -1 : (a->j > b->j ? 1 : 0);", "return a->j > b->j ? -1 : (a->j < b->j ? 1 : 0);"),
+    ("first_position_not_raised", "Sp[0] = mx;", "(void)mx;"),
+    ("partial_argmax_over_selected", "if (!sel[t] && (c < 0 || Sp[t] > Sp[c])) c = t;", "if (c < 0 || Sp[t] > Sp[c]) c = t;"),
+    ("partial_takes_span_start", "near[n].dist = t > c ? t - c : c - t;", "near[n].dist = t;"),
+    ("nearest_tie_to_higher_index", "return a->t < b->t ? -1 : (a->t > b->t ? 1 : 0);", "return a->t > b->t ? -1 : (a->t < b->t ? 1 : 0);"),
+    ("latent_tail_off_by_one", "if (t < n_sink || t >= T - n_latent) { sel[t] = 1; ++count; }", "if (t < n_sink || t > T - n_latent) { sel[t] = 1; ++count; }"),
+    ("short_span_mean_over_full_width", "rank[j].mean = acc / (double)(hi - lo);", "rank[j].mean = acc / (double)span_w;"),
+    ("short_span_mean_over_full_width_f32", "rank[j].mean = (double)(acc / (float)(hi - lo));", "rank[j].mean = (double)(acc / (float)span_w);"),
+    ("ranking_ascending", "if (a->mean > b->mean) return -1;\n    if (a->mean < b->mean) return 1;", "if (a->mean < b->mean) return -1;\n    if (a->mean > b->mean) return 1;"),
+    ("compact_offset_dropped", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + (off + j) * d;", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + j * d;"),
+    ("compact_v_from_k", "memcpy(v_out + dst, V + src, sizeof(uint16_t) * (size_t)d);", "memcpy(v_out + dst, K + src, sizeof(uint16_t) * (size_t)d);"),
+]
+
+
+def _build(args):
+    name, old, new, src, outdir = args
+    if src.count(old) != 1:
+        return name, None, "snippet occurs %d times" % src.count(old)
+    path = os.path.join(outdir, name + ".c")
+    with open(path, "w") as f:
+        f.write(src.replace(old, new))
+    so = os.path.join(outdir, "lib_" + name + ".so")
+    oracle.build(path, so, force=True)
+    return name, so, None
+
+
+@pytest.fixture(scope="module")
+def mutant_libs():
+    with open(oracle._SRC) as f:
+        src = f.read()
+    outdir = tempfile.mkdtemp(prefix="cbo_mutants_")
+    with cf.ThreadPoolExecutor(max_workers=os.cpu_count() or 4) as ex:
+        res = list(ex.map(_build, [(n, o, nw, src, outdir) for n, o, nw in MUTANTS]))
+    return {n: (so, err) for n, so, err in res}
+
+
+@pytest.mark.parametrize("name", [m[0] for m in MUTANTS])
+def test_mutant_is_caught(mutant_libs, name):
+    so, err = mutant_libs[name]
+    assert err is None, err
+    o = oracle.Oracle(so)
+    caught = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(o)
+        except (AssertionError, RuntimeError, ValueError):
+            caught.append(pin.__name__)
+    assert caught, "no pin catches the planted mistake %r" % name
