@@ -1,0 +1,414 @@
+"""Benchmark of the CacheBack score -> select -> compact path on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+
+One step = score + select + compact of every sender of the workload (default:
+the Qwen3-8B-shaped single sender, T = 8192, m = 64, keep 25%) with inputs
+resident in HBM; the K/V inputs (1.2 GB) are larger than L2, so no flush is
+needed between steps.  Prints one JSON line (rank 0).  Under torchrun each
+rank runs its own replica (independent senders, no collective) and `value` is
+the tokens of all ranks / the slowest rank's time.
+
+--impl reference times the CPU oracle (the fp64 C restatement in oracle/) on
+the host cores, on a bounded sample of the same workload, scaled to the metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "sender KV tokens scored+compacted/s; achieved HBM GB/s vs GB300 peak"
+UNIT = "tokens/s"
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def workload_bytes_flops(spec, keep):
+    """Algorithmic traffic and tensor flops of one step.
+
+    bytes: K read once by the score (the second logit pass re-reads it, counted as
+    algorithmically unnecessary) + compaction reads and writes of the kept K and V
+    rows.  flops: two QK^T passes (statistics, then normalised accumulation).
+    """
+    sh = spec.shape
+    tot_b = 0
+    tot_f = 0
+    score_b = 0
+    compact_b = 0
+    for i in range(spec.n_senders):
+        T = spec.T[i % len(spec.T)]
+        B = min(T, max(0, math.ceil(keep * T)))
+        row = sh.head_dim * 2
+        kbytes = sh.n_layers * sh.n_kv_heads * T * row
+        cbytes = 2 * 2 * sh.n_layers * sh.n_kv_heads * B * row   # read + write, K and V
+        score_b += kbytes
+        compact_b += cbytes
+        tot_f += 2 * 2 * spec.m * sh.n_q_heads * T * sh.head_dim * sh.n_layers
+    tot_b = score_b + compact_b
+    return tot_b, score_b, compact_b, tot_f
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled in the background."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.samples = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+
+    def summary(self, t0, t1):
+        rows = []
+        for ts, line in self.samples:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            rows.append((ts, parts))
+        window = [r for r in rows if t0 <= r[0] <= t1]
+        note = "in timed region"
+        if not window:
+            # the timed region was shorter than the sampling period: take the samples nearest it
+            window = sorted(rows, key=lambda r: min(abs(r[0] - t0), abs(r[0] - t1)))[:3]
+            note = "nearest samples (timed region shorter than the 50 ms sampling period)"
+        if not window:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(p[1]) for _, p in window if num(p[1]) is not None]
+        smax = [num(p[2]) for _, p in window if num(p[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for _, p in window for k in range(4) if p[5 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(window), "note": note,
+                "power_w_max": max((num(p[3]) or 0.0) for _, p in window)}
+
+
+def dist_init():
+    import torch
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(ws, x: float) -> float:
+    if ws <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the cpu_baseline object and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(spec_name: str, n_layers_sample: int, seed: int = 0):
+    """Time the oracle on sender 0 of the workload, scoring n_layers_sample of its layers.
+
+    Scoring is linear in the scored layers, so the full-workload time is the sample's
+    score time x (layers / sampled layers) x senders, plus select and compact times x senders.
+    """
+    import oracle
+    import synth
+    spec = synth.SPECS[spec_name]
+    o = oracle.default()
+    snd = synth.make_sender(spec, seed, 0, synth.make_query(spec, seed, 0, "cpu"), "cpu")
+    Q = synth.make_query(spec, seed, 0, "cpu")
+    nl = min(n_layers_sample, spec.shape.n_layers)
+    keep = spec.keeps[len(spec.keeps) // 2] if len(spec.keeps) > 1 else spec.keeps[0]
+    t0 = time.perf_counter()
+    r = o.score(snd.K[:nl].contiguous(), Q[:nl].contiguous())
+    t1 = time.perf_counter()
+    B = oracle.budget(snd.T, keep)
+    idx = o.select(r["S"], B)
+    t2 = time.perf_counter()
+    o.compact(snd.K, snd.V, idx)
+    t3 = time.perf_counter()
+    per_sender = (t1 - t0) * spec.shape.n_layers / nl + (t2 - t1) + (t3 - t2)
+    total_tokens = sum(spec.T[i % len(spec.T)] for i in range(spec.n_senders))
+    total_time = per_sender * spec.n_senders * (total_tokens / spec.n_senders) / snd.T
+    return {
+        "value": total_tokens / total_time,
+        "unit": UNIT,
+        "cores": o.max_threads(),
+        "kind": "oracle",
+        "sample": "sender 0 of %s: score on %d of %d layers (x%.1f), full select and compact, scaled to %d "
+                  "sender(s); fp64 C oracle, OpenMP over KV-head groups" % (
+                      spec_name, nl, spec.shape.n_layers, spec.shape.n_layers / nl, spec.n_senders),
+        "seconds": {"score_sample": t1 - t0, "select": t2 - t1, "compact": t3 - t2},
+    }
+
+
+def run_reference(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    vals = []
+    for k in range(args.warmup + args.steps):
+        r = oracle_sample(args.workload, 1)
+        if k >= args.warmup:
+            vals.append(r)
+    v = statistics.median([x["value"] for x in vals])
+    per_step_s = None
+    import synth
+    spec = synth.SPECS[args.workload]
+    tokens = sum(spec.T[i % len(spec.T)] for i in range(spec.n_senders))
+    per_step_s = tokens / v
+    cpu = dict(vals[0])
+    cpu["value"] = v
+    cpu.pop("seconds", None)
+    out = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": per_step_s * 1e3, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": args.workload, "keep": spec.keeps[0], "senders": spec.n_senders},
+           "cpu_baseline": cpu,
+           "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    import paper_2609_32046_gb300 as cb
+    import synth
+    ws, rank, local = dist_init()
+    spec = synth.SPECS[args.workload]
+    keep = args.keep if args.keep is not None else spec.keeps[0]
+    dev = torch.device("cuda", local)
+    w = synth.make_workload(args.workload, seed=rank, device=dev)
+    senders = [(s.K, s.V) for s in w.senders]
+    queries = [w.queries[s.task] for s in w.senders]
+    c = cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads, spec.shape.head_dim,
+                     spec.m, max(spec.T), len(senders))
+    f = cb.Filter(c, senders, queries, keep, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    n_launch_per_step = 6 * math.ceil(len(senders) / 64)
+
+    for _ in range(args.warmup):
+        f.run(stream)
+    c.sync_status(stream)
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4 * args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.15)
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    t_wall0 = time.time()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for k in range(args.steps):
+        ev[4 * k].record(stream)
+        f.score(stream)
+        ev[4 * k + 1].record(stream)
+        f.select(stream)
+        ev[4 * k + 2].record(stream)
+        f.compact(stream)
+        ev[4 * k + 3].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    barrier(ws)
+    sampler.stop()
+    c.sync_status(stream)
+    ms = start.elapsed_time(end)
+    ms_max = max_over_ranks(ws, ms)
+    per = {"score": [], "select": [], "compact": []}
+    for k in range(args.steps):
+        per["score"].append(ev[4 * k].elapsed_time(ev[4 * k + 1]))
+        per["select"].append(ev[4 * k + 1].elapsed_time(ev[4 * k + 2]))
+        per["compact"].append(ev[4 * k + 2].elapsed_time(ev[4 * k + 3]))
+    avg = {k: sum(v) / len(v) for k, v in per.items()}
+
+    tokens_per_rank = sum(f.Ts)
+    value = tokens_per_rank * ws * args.steps / (ms_max / 1e3)
+    hbm_peak, tc_peak, tc_sus, src = peaks()
+    tot_b, score_b, compact_b, flops = workload_bytes_flops(spec, keep)
+    step_s = ms / args.steps / 1e3
+
+    # e2e: the same step through the C-ABI with the inputs in pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        hK = [K.cpu().pin_memory() for K, _ in senders]
+        hV = [V.cpu().pin_memory() for _, V in senders]
+        hQ = [q.cpu().pin_memory() for q in w.queries]
+        hko = torch.empty(f.k_out.shape, dtype=f.k_out.dtype).pin_memory()
+        hvo = torch.empty_like(hko).pin_memory()
+        hidx = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in f.idx]
+        h2d = sum(x.numel() * x.element_size() for x in hK + hV + hQ)
+        d2h = hko.numel() * 2 * 2 + sum(x.numel() * 4 for x in hidx)
+
+        def e2e_step():
+            for (K, V), hk, hv in zip(senders, hK, hV):
+                K.copy_(hk, non_blocking=True)
+                V.copy_(hv, non_blocking=True)
+            for q, hq in zip(w.queries, hQ):
+                q.copy_(hq, non_blocking=True)
+            f.run(stream)
+            hko.copy_(f.k_out, non_blocking=True)
+            hvo.copy_(f.v_out, non_blocking=True)
+            for x, hx in zip(f.idx, hidx):
+                hx.copy_(x, non_blocking=True)
+
+        n_e2e = max(2, min(args.steps, 5))
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier(ws)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(ws)
+        ems = max_over_ranks(ws, e0.elapsed_time(e1))
+        e2e = {"value": tokens_per_rank * ws * n_e2e / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": n_e2e,
+               "ms_per_step": ems / n_e2e}
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "senders": len(senders), "T": list(spec.T[:3]), "m": spec.m,
+                   "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
+                   "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": keep,
+                   "l2": "inputs larger than L2 (K+V %.2f GB per rank), no flush" % (
+                       sum(K.numel() * 4 for K, _ in senders) / 1e9),
+                   "parallelism": "replicas" if ws > 1 else "single"},
+        "hbm_gbs": tot_b / step_s / 1e9,
+        "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
+        "algorithmic_bytes_per_step": tot_b,
+        "step_ms": {k: v for k, v in avg.items()},
+        "roofline": {
+            "bound": "tensor", "kernel": "score (stats + accumulate passes)",
+            "achieved": flops / (avg["score"] / 1e3) / 1e12, "peak": tc_peak, "unit": "TFLOP/s",
+            "frac": flops / (avg["score"] / 1e3) / 1e12 / tc_peak, "traffic": None,
+            "peak_source": "%s bf16 burst" % src,
+        },
+        "roofline_compact": {
+            "bound": "hbm", "achieved": compact_b / (avg["compact"] / 1e3) / 1e9, "peak": hbm_peak, "unit": "GB/s",
+            "frac": compact_b / (avg["compact"] / 1e3) / 1e9 / hbm_peak, "peak_source": "%s copy" % src,
+        },
+        "gpu_launches": n_launch_per_step * args.steps,
+        "clocks": sampler.summary(t_wall0, t_wall1),
+    }
+    if e2e:
+        out["e2e"] = e2e
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        out["cpu_baseline"] = oracle_sample(args.workload, args.cpu_layers)
+    if rank == 0:
+        print(json.dumps(out))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="qwen8b")
+    ap.add_argument("--keep", type=float, default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-layers", type=int, default=4)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    from paper_2609_32046_gb300.build import build, up_to_date, LIB_PATH
+    if int(os.environ.get("LOCAL_RANK", "0")) == 0:
+        build()
+    else:
+        for _ in range(600):
+            if up_to_date():
+                break
+            time.sleep(0.5)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,175 @@
+/*
+ * cacheback.h -- C-ABI of the GB300 (sm_103a) CacheBack filtering path:
+ * score every cached sender position by the attention it receives from the
+ * receiver's query, select positions under a keep budget, and gather the
+ * selected K/V rows of every layer into one contiguous send buffer.
+ *
+ * Paper: receiver-conditioned communication with CacheBack.
+ *   App. A (formal model): the sender cache M_S = {(K_j^l, V_j^l)}, l = 1..L, j = 1..N.
+ *   App. C.1 (general scoring rule): attention a_{l,h,r,t} from the m query tokens,
+ *     mean query attention Q_t, the CacheBack correction C_{p,t}, Pool_7.
+ *   App. D.2 (parameter sensitivity): S_t(p, alpha) = Q_t * C_{p,t}^alpha
+ *     (CacheBack: p = alpha = 2; alpha = 0 is mean query attention).
+ *   App. C.2 (budgets and position selection): B_i = ceil(T_i / r), forced
+ *     first and latent positions, width-16 span ranking, source-order output.
+ *
+ * Conventions shared by every entry point
+ *   - All data pointers inside descriptors are DEVICE pointers owned by the
+ *     caller; arrays of descriptors / pointers / sizes passed directly are HOST
+ *     arrays read during the call only.  The library never frees caller memory.
+ *   - K, V and Q are bf16 (raw 16-bit storage).  Strides are in ELEMENTS; the
+ *     head-dimension stride is 1.  Every device pointer must be 16-byte aligned
+ *     and every stride a multiple of 8 elements.
+ *   - Calls are asynchronous on the given CUDA stream (a cudaStream_t passed
+ *     as void*; NULL is the legacy default stream).  Errors found on the host
+ *     are returned synchronously and nothing is enqueued.  cb_last_error()
+ *     describes the most recent failure of that context.
+ *   - Results are bitwise deterministic: every reduction has a fixed order.
+ *   - Query head h reads KV head h / G, G = n_q_heads / n_kv_heads (App. C.1:
+ *     query heads that share each KV head).
+ *   - A context is not thread-safe: one host thread at a time.  Scratch is
+ *     shared by calls on one context, so calls on one context must be ordered
+ *     on one stream (or synchronised); use one context per concurrent stream.
+ */
+#ifndef CACHEBACK_H_
+#define CACHEBACK_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CB_OK = 0,
+    CB_EINVAL = 1,   /* null / misaligned pointer, bad parameter value */
+    CB_ESHAPE = 2,   /* unsupported or inconsistent shape, above a creation limit */
+    CB_EBUDGET = 3,  /* budget below the forced positions, above T, or beyond the output capacity */
+    CB_ENOMEM = 4,   /* device allocation failed */
+    CB_ECUDA = 5,    /* a CUDA runtime call or a kernel launch failed */
+    CB_ETIMEOUT = 6, /* reserved: a bounded device wait gave up */
+    CB_EDEVICE = 7   /* a kernel's own bounds check rejected an input (see cb_sync_status) */
+} cb_status;
+
+typedef struct cb_ctx cb_ctx; /* opaque; owns device scratch only */
+
+/*
+ * Creation-time configuration (App. C.1 notation).
+ *   n_layers           |L|: scored layers only (global-attention layers; App. C.1 skips
+ *                      local/sliding layers, App. F lists 8/48 for Gemma, 6/62 for Nemotron)
+ *   n_q_heads          Hq, query heads per layer
+ *   n_kv_heads         Hkv; Hq % Hkv == 0 and G = Hq / Hkv in {1, 2, 4}
+ *   head_dim           d in {64, 128}
+ *   max_query_tokens   upper bound on m (1..1024)
+ *   max_positions      upper bound on any sender's T (scratch is sized from it)
+ *   max_senders        upper bound on senders per call
+ *   softmax_scale      logit scale; 0 selects 1/sqrt(d)
+ *   p, alpha           correction power p > 1 and strength alpha >= 0 (App. D.2)
+ *   pool_width         Pool window, odd, 1..15 (7 in the paper; 1 disables pooling)
+ *   span_width         span width for selection, 1..256 (16 in the paper; 1 ranks positions)
+ *   n_sink, n_latent   forced positions: the first n_sink and the last n_latent (1 and 40)
+ */
+typedef struct {
+    int32_t n_layers, n_q_heads, n_kv_heads, head_dim;
+    int32_t max_query_tokens;
+    int64_t max_positions;
+    int32_t max_senders;
+    float softmax_scale;
+    float p, alpha;
+    int32_t pool_width;
+    int32_t span_width;
+    int32_t n_sink, n_latent;
+} cb_config;
+
+/* One sender's cache M_S (App. A): K[l][g][t][:] at k + l*s_layer + g*s_head + t*s_pos,
+ * V likewise with the same strides.  T = number of cached positions (T_i = H_i + G_i, Sec. 2). */
+typedef struct {
+    const void *k, *v;
+    int64_t T;
+    int64_t s_layer, s_head, s_pos;
+} cb_kv;
+
+/* The receiver query's post-RoPE query vectors in the sender's scored layers (Sec. 3:
+ * the sender appends q and computes only the query tokens against its cache):
+ * Q[l][r][h][:] at q + l*s_layer + r*s_tok + h*s_head, r < m.  Several senders may share one. */
+typedef struct {
+    const void *q;
+    int32_t m;
+    int64_t s_layer, s_tok, s_head;
+} cb_query;
+
+/* Fill *cfg with the paper's defaults (p = alpha = 2, Pool_7, width-16 spans, 1 sink,
+ * 40 latent positions, scale 1/sqrt(d)) and zero shapes / limits. */
+void cb_config_init(cb_config *cfg);
+
+/* Validate cfg, select the current CUDA device, and allocate the scratch the limits need.
+ * On success *out owns the scratch until cb_destroy.  Errors: CB_EINVAL, CB_ESHAPE, CB_ENOMEM,
+ * CB_ECUDA (then *out is NULL). */
+cb_status cb_create(const cb_config *cfg, cb_ctx **out);
+
+/*
+ * Score (App. C.1, App. D.2): for each sender i, write scores[i][t], t < T_i (fp32, device):
+ *   S_t = Q_t * C_{p,t}^alpha,
+ *   Q_t = Pool( sum_l 1/(m Hq) sum_r sum_h a_{l,h,r,t} ),
+ *   C_{p,t} = ( sum_s mean_r Pool(b_{s,r,.})_t^p / sum_s Pool(mean_r b_{s,r,.})_t^p )^(1/(p-1)),
+ * a = softmax over the sender's T positions of softmax_scale * <q_{l,r,h}, k_{l,h/G,t}>,
+ * b_{s,r,t} = mean of a over the G query heads of KV group s = (l, g); C = 1 where the
+ * denominator is 0 (or below FLT_MIN in fp32).  Sender i is scored against queries[i].
+ *   n         1..max_senders;  senders, queries, scores: host arrays of n entries
+ *   scores[i] device float[T_i], written; 16-byte aligned
+ * Errors: CB_EINVAL (null/misaligned pointers, strides), CB_ESHAPE (T_i or m_i above the limits).
+ */
+cb_status cb_score(cb_ctx *ctx, int32_t n, const cb_kv *senders, const cb_query *queries,
+                   float *const *scores, void *stream);
+
+/* B = ceil(keep * T) computed in double, clamped to [0, T] (App. C.2: B_i = ceil(T_i / r)
+ * with keep = 1/r).  Pure host function; needs no context. */
+int64_t cb_budget(int64_t T, double keep);
+
+/*
+ * Select (App. C.2): for each sender i, write idx[i][0..budget[i]) (int32, device),
+ * strictly ascending, containing the forced positions (the first n_sink and the last
+ * n_latent) and filled from spans ranked by mean score after the first position's score
+ * is raised to the maximum; equal means favour the earlier span; a span that does not
+ * fit contributes its unselected positions nearest its highest-scoring one (ties: lower index).
+ * Span means are formed in fp32 in index order and divided by the span's own length.
+ *   scores[i]  device float[T[i]] (e.g. cb_score's output)
+ *   T, budget  host int64 arrays of n entries; min(T, n_sink + n_latent) <= budget[i] <= T[i]
+ *   idx[i]     device int32[budget[i]], written
+ * Errors: CB_EINVAL, CB_ESHAPE (T above max_positions), CB_EBUDGET.
+ */
+cb_status cb_select(cb_ctx *ctx, int32_t n, const float *const *scores, const int64_t *T,
+                    const int64_t *budget, int32_t *const *idx, void *stream);
+
+/*
+ * Compact (the message of selected positions; Sec. 3 "State Representation", App. C.3):
+ * for every sender i, layer l, KV head g and j < budget[i]:
+ *   k_out[l*o_layer + g*o_head + (out_offset[i] + j)*d .. +d) = K_i[l][g][idx[i][j]][:]
+ * and likewise v_out from V_i -- a bit-exact copy.  Fan-in senders are concatenated by
+ * giving each its own out_offset.  out_capacity is the number of position rows per
+ * (l, g) in the output; out_offset[i] + budget[i] <= out_capacity is required.
+ * Indices outside [0, T_i) are skipped by the kernel and reported as CB_EDEVICE by the
+ * next cb_sync_status().
+ * Errors: CB_EINVAL, CB_ESHAPE, CB_EBUDGET (capacity overflow).
+ */
+cb_status cb_compact(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t *const *idx,
+                     const int64_t *budget, void *k_out, void *v_out, int64_t out_capacity,
+                     const int64_t *out_offset, int64_t o_layer, int64_t o_head, void *stream);
+
+/* Wait for `stream`, then report (and clear) errors the kernels recorded on the device
+ * (CB_EDEVICE) or a failed launch (CB_ECUDA).  Blocks the host. */
+cb_status cb_sync_status(cb_ctx *ctx, void *stream);
+
+/* Free the context's scratch (after synchronising its device).  NULL is ignored. */
+void cb_destroy(cb_ctx *ctx);
+
+/* Text of the context's most recent error ("" if none).  NULL ctx: the last cb_create failure. */
+const char *cb_last_error(const cb_ctx *ctx);
+
+/* Device scratch bytes the context holds (for capacity planning). */
+int64_t cb_scratch_bytes(const cb_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CACHEBACK_H_ */

@@ -1,0 +1,69 @@
+"""GB300-native CacheBack receiver-conditioned KV filtering.
+
+    score   (App. C.1, App. D.2)  every cached sender position by the attention it
+            receives from the receiver's query tokens: S_t = Q_t * C_{p,t}^alpha
+    select  (App. C.2)            B = ceil(keep * T) positions by the span rule
+    compact                       the selected K/V rows of every layer into one
+                                  contiguous send buffer (fan-in senders concatenated)
+
+The compute runs in hand-written sm_103a CUDA kernels behind the C-ABI of
+include/cacheback.h (libcacheback.so); this package is the Python binding.
+"""
+from __future__ import annotations
+
+from typing import List, Optional, Sequence
+
+from .binding import (CB_EBUDGET, CB_ECUDA, CB_EDEVICE, CB_EINVAL, CB_ENOMEM, CB_ESHAPE, CB_OK, EXPORTED,
+                      LIB_PATH, CacheBack, CBError, budget, load_library)
+
+__all__ = ["CacheBack", "CBError", "budget", "load_library", "LIB_PATH", "EXPORTED", "Filter",
+           "CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_EDEVICE"]
+
+
+class Filter:
+    """Score -> select -> compact for a fixed batch of senders, outputs allocated once.
+
+    senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors
+    queries: list of Q bf16 [nL][m_i][Hq][d] device tensors, one per sender (may repeat)
+    keep:    keep ratio; budgets B_i = ceil(keep * T_i)
+    The send buffer holds every sender's rows back to back: sender i at offset sum_{j<i} B_j.
+    """
+
+    def __init__(self, cb: CacheBack, senders: Sequence, queries: Sequence, keep: float, device=None):
+        import torch
+        self.cb = cb
+        self.Ks = [k for k, _ in senders]
+        self.Vs = [v for _, v in senders]
+        self.Qs = list(queries)
+        dev = device or self.Ks[0].device
+        self.Ts = [int(K.shape[2]) for K in self.Ks]
+        self.budgets = [budget(T, keep) for T in self.Ts]
+        self.offsets = []
+        off = 0
+        for b in self.budgets:
+            self.offsets.append(off)
+            off += b
+        self.capacity = off
+        nL, Hkv, _, d = self.Ks[0].shape
+        self.scores = [torch.empty(T, dtype=torch.float32, device=dev) for T in self.Ts]
+        self.idx = [torch.empty(max(b, 1), dtype=torch.int32, device=dev) for b in self.budgets]
+        self.k_out = torch.empty(nL, Hkv, max(self.capacity, 1), d, dtype=self.Ks[0].dtype, device=dev)
+        self.v_out = torch.empty_like(self.k_out)
+
+    def score(self, stream=None):
+        self.cb.score(self.Ks, self.Qs, self.scores, stream)
+
+    def select(self, stream=None):
+        self.cb.select(self.scores, self.Ts, self.budgets, self.idx, stream)
+
+    def compact(self, stream=None):
+        self.cb.compact(self.Ks, self.Vs, self.idx, self.budgets, self.k_out, self.v_out, self.offsets, stream)
+
+    def run(self, stream=None):
+        self.score(stream)
+        self.select(stream)
+        self.compact(stream)
+        return self
+
+    def indices(self) -> List:
+        return [x[:b] for x, b in zip(self.idx, self.budgets)]

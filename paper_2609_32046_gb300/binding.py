@@ -1,0 +1,196 @@
+"""Thin Python binding of include/cacheback.h (argument marshalling only).
+
+Every step of the path runs in libcacheback.so's CUDA kernels; this module only
+turns torch tensors into pointers, sizes and strides.  If the library is missing
+the import of `CacheBack` fails loudly: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from typing import Optional, Sequence
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libcacheback.so")
+
+CB_OK, CB_EINVAL, CB_ESHAPE, CB_EBUDGET, CB_ENOMEM, CB_ECUDA, CB_ETIMEOUT, CB_EDEVICE = range(8)
+STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_ETIMEOUT",
+                "CB_EDEVICE"]
+
+# Every entry point include/cacheback.h declares (checked by the tests).
+EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
+            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes"]
+
+
+class CBError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        name = STATUS_NAMES[status] if 0 <= status < len(STATUS_NAMES) else str(status)
+        super().__init__("%s: %s" % (name, message))
+        self.status = status
+
+
+class cb_config(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("max_query_tokens", ctypes.c_int32),
+                ("max_positions", ctypes.c_int64), ("max_senders", ctypes.c_int32),
+                ("softmax_scale", ctypes.c_float), ("p", ctypes.c_float), ("alpha", ctypes.c_float),
+                ("pool_width", ctypes.c_int32), ("span_width", ctypes.c_int32),
+                ("n_sink", ctypes.c_int32), ("n_latent", ctypes.c_int32)]
+
+
+class cb_kv(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("T", ctypes.c_int64),
+                ("s_layer", ctypes.c_int64), ("s_head", ctypes.c_int64), ("s_pos", ctypes.c_int64)]
+
+
+class cb_query(ctypes.Structure):
+    _fields_ = [("q", ctypes.c_void_p), ("m", ctypes.c_int32), ("s_layer", ctypes.c_int64),
+                ("s_tok", ctypes.c_int64), ("s_head", ctypes.c_int64)]
+
+
+_LIB = None
+
+
+def load_library(path: Optional[str] = None) -> ctypes.CDLL:
+    """Load libcacheback.so (built by paper_2609_32046_gb300.build); raises if absent."""
+    global _LIB
+    if _LIB is not None and path is None:
+        return _LIB
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise ImportError("libcacheback.so is not built (%s); run `python -m paper_2609_32046_gb300.build` "
+                          "or __graft_entry__.build()" % p)
+    lib = ctypes.CDLL(p)
+    P = ctypes.c_void_p
+    lib.cb_config_init.argtypes = [ctypes.POINTER(cb_config)]
+    lib.cb_config_init.restype = None
+    lib.cb_create.argtypes = [ctypes.POINTER(cb_config), ctypes.POINTER(P)]
+    lib.cb_create.restype = ctypes.c_int
+    lib.cb_score.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), ctypes.POINTER(cb_query), P, P]
+    lib.cb_score.restype = ctypes.c_int
+    lib.cb_budget.argtypes = [ctypes.c_int64, ctypes.c_double]
+    lib.cb_budget.restype = ctypes.c_int64
+    lib.cb_select.argtypes = [P, ctypes.c_int32, P, P, P, P, P]
+    lib.cb_select.restype = ctypes.c_int
+    lib.cb_compact.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), P, P, P, P, ctypes.c_int64, P,
+                               ctypes.c_int64, ctypes.c_int64, P]
+    lib.cb_compact.restype = ctypes.c_int
+    lib.cb_sync_status.argtypes = [P, P]
+    lib.cb_sync_status.restype = ctypes.c_int
+    lib.cb_destroy.argtypes = [P]
+    lib.cb_destroy.restype = None
+    lib.cb_last_error.argtypes = [P]
+    lib.cb_last_error.restype = ctypes.c_char_p
+    lib.cb_scratch_bytes.argtypes = [P]
+    lib.cb_scratch_bytes.restype = ctypes.c_int64
+    if path is None:
+        _LIB = lib
+    return lib
+
+
+def budget(T: int, keep: float) -> int:
+    """ceil(keep * T) in double, clamped to [0, T] (App. C.2), computed by the library."""
+    return int(load_library().cb_budget(int(T), float(keep)))
+
+
+def _ptr_array(values, ctype=ctypes.c_void_p):
+    arr = (ctype * len(values))(*values)
+    return arr
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def kv_desc(K, V=None) -> cb_kv:
+    """K, V: bf16 [nL][Hkv][T][d] (any strides with unit head-dim stride)."""
+    assert K.dtype.itemsize == 2 and K.stride(3) == 1
+    if V is not None:
+        assert V.shape == K.shape and V.stride() == K.stride()
+    return cb_kv(K.data_ptr(), V.data_ptr() if V is not None else None, K.shape[2],
+                 K.stride(0), K.stride(1), K.stride(2))
+
+
+def query_desc(Q) -> cb_query:
+    """Q: bf16 [nL][m][Hq][d]."""
+    assert Q.dtype.itemsize == 2 and Q.stride(3) == 1
+    return cb_query(Q.data_ptr(), Q.shape[1], Q.stride(0), Q.stride(1), Q.stride(2))
+
+
+class CacheBack:
+    """One cb_ctx.  Methods enqueue work on a CUDA stream (default: torch's current stream)."""
+
+    def __init__(self, n_layers: int, n_q_heads: int, n_kv_heads: int, head_dim: int, max_query_tokens: int,
+                 max_positions: int, max_senders: int = 1, p: float = 2.0, alpha: float = 2.0,
+                 pool_width: int = 7, span_width: int = 16, n_sink: int = 1, n_latent: int = 40,
+                 softmax_scale: float = 0.0, lib_path: Optional[str] = None):
+        self.lib = load_library(lib_path)
+        cfg = cb_config()
+        self.lib.cb_config_init(ctypes.byref(cfg))
+        cfg.n_layers, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim = n_layers, n_q_heads, n_kv_heads, head_dim
+        cfg.max_query_tokens, cfg.max_positions, cfg.max_senders = max_query_tokens, max_positions, max_senders
+        cfg.softmax_scale, cfg.p, cfg.alpha = softmax_scale, p, alpha
+        cfg.pool_width, cfg.span_width, cfg.n_sink, cfg.n_latent = pool_width, span_width, n_sink, n_latent
+        self.cfg = cfg
+        h = ctypes.c_void_p()
+        st = self.lib.cb_create(ctypes.byref(cfg), ctypes.byref(h))
+        if st != CB_OK:
+            raise CBError(st, self.lib.cb_last_error(None).decode())
+        self.h = h
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.cb_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, st: int):
+        if st != CB_OK:
+            raise CBError(st, self.lib.cb_last_error(self.h).decode())
+
+    @property
+    def scratch_bytes(self) -> int:
+        return int(self.lib.cb_scratch_bytes(self.h))
+
+    # -- the three steps ----------------------------------------------------
+    def score(self, Ks: Sequence, Qs: Sequence, scores: Sequence, stream=None):
+        n = len(Ks)
+        kv = (cb_kv * n)(*[kv_desc(K) for K in Ks])
+        qq = (cb_query * n)(*[query_desc(Q) for Q in Qs])
+        out = _ptr_array([s.data_ptr() for s in scores])
+        self._check(self.lib.cb_score(self.h, n, kv, qq, out, _stream_handle(stream)))
+
+    def select(self, scores: Sequence, Ts: Sequence[int], budgets: Sequence[int], idx: Sequence, stream=None):
+        n = len(scores)
+        sp = _ptr_array([s.data_ptr() for s in scores])
+        Ta = _ptr_array([int(t) for t in Ts], ctypes.c_int64)
+        Ba = _ptr_array([int(b) for b in budgets], ctypes.c_int64)
+        ip = _ptr_array([x.data_ptr() for x in idx])
+        self._check(self.lib.cb_select(self.h, n, sp, Ta, Ba, ip, _stream_handle(stream)))
+
+    def compact(self, Ks: Sequence, Vs: Sequence, idx: Sequence, budgets: Sequence[int], k_out, v_out,
+                offsets: Sequence[int], stream=None):
+        """k_out, v_out: bf16 [nL][Hkv][capacity][d] (contiguous rows)."""
+        n = len(Ks)
+        kv = (cb_kv * n)(*[kv_desc(K, V) for K, V in zip(Ks, Vs)])
+        ip = _ptr_array([x.data_ptr() for x in idx])
+        Ba = _ptr_array([int(b) for b in budgets], ctypes.c_int64)
+        Oa = _ptr_array([int(o) for o in offsets], ctypes.c_int64)
+        assert k_out.stride(3) == 1 and k_out.stride(2) == k_out.shape[3] and v_out.stride() == k_out.stride()
+        self._check(self.lib.cb_compact(self.h, n, kv, ip, Ba, k_out.data_ptr(), v_out.data_ptr(),
+                                        k_out.shape[2], Oa, k_out.stride(0), k_out.stride(1),
+                                        _stream_handle(stream)))
+
+    def sync_status(self, stream=None):
+        self._check(self.lib.cb_sync_status(self.h, _stream_handle(stream)))

@@ -1,0 +1,404 @@
+// C-ABI of the CacheBack filtering path (declared in include/cacheback.h).
+// Host-side validation, scratch ownership and launch plumbing; every step of
+// the path itself runs in the kernels of cb_score.cu, cb_select.cu and
+// cb_compact.cu.
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "cacheback.h"
+#include "cb_internal.cuh"
+
+struct cb_ctx {
+    cb_config cfg;
+    int device = 0;
+    int num_sms = 0;
+    int G = 1;
+    float scale = 0.f;
+    int64_t n_chunk1_max = 0;
+    float2* stats = nullptr;
+    float* offs = nullptr;
+    float* part = nullptr;
+    float* span_keys = nullptr;
+    uint32_t* err = nullptr;
+    int64_t keys_per_sender = 0;
+    int64_t scratch_bytes = 0;
+    std::string last_error;
+};
+
+namespace {
+
+thread_local std::string g_create_error;
+
+cb_status fail(cb_ctx* ctx, cb_status st, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (ctx)
+        ctx->last_error = buf;
+    else
+        g_create_error = buf;
+    return st;
+}
+
+// Makes ctx's device current for the duration of a call, restoring the caller's device after.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) { ok = false; return; }
+        if (prev != dev && cudaSetDevice(dev) != cudaSuccess) ok = false;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The pointer must be device (or managed) memory on ctx's device.
+cb_status check_device_ptr(cb_ctx* ctx, const void* p, const char* what, int i) {
+    if (!p) return fail(ctx, CB_EINVAL, "%s[%d] is NULL", what, i);
+    if (!aligned16(p)) return fail(ctx, CB_EINVAL, "%s[%d] is not 16-byte aligned", what, i);
+    cudaPointerAttributes a;
+    cudaError_t e = cudaPointerGetAttributes(&a, p);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ctx, CB_EINVAL, "%s[%d]: cannot query pointer (%s)", what, i, cudaGetErrorString(e));
+    }
+    if (a.type == cudaMemoryTypeManaged) return CB_OK;
+    if (a.type != cudaMemoryTypeDevice)
+        return fail(ctx, CB_EINVAL, "%s[%d] is not device memory", what, i);
+    if (a.device != ctx->device)
+        return fail(ctx, CB_EINVAL, "%s[%d] lives on device %d, context on device %d", what, i, a.device,
+                    ctx->device);
+    return CB_OK;
+}
+
+bool stride_ok(int64_t s) { return s > 0 && (s % 8) == 0; }
+
+template <typename T>
+cudaError_t alloc(T** p, size_t count, int64_t* total) {
+    if (count == 0) count = 1;
+    *total += (int64_t)(count * sizeof(T));
+    return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+}
+
+}  // namespace
+
+extern "C" {
+
+void cb_config_init(cb_config* cfg) {
+    if (!cfg) return;
+    std::memset(cfg, 0, sizeof *cfg);
+    cfg->softmax_scale = 0.f;
+    cfg->p = 2.f;
+    cfg->alpha = 2.f;
+    cfg->pool_width = 7;
+    cfg->span_width = 16;
+    cfg->n_sink = 1;
+    cfg->n_latent = 40;
+    cfg->max_senders = 1;
+}
+
+int64_t cb_budget(int64_t T, double keep) {
+    if (T <= 0 || !(keep > 0.0)) return 0;
+    const double b = std::ceil(keep * (double)T);
+    if (b >= (double)T) return T;
+    return (int64_t)b;
+}
+
+const char* cb_last_error(const cb_ctx* ctx) { return ctx ? ctx->last_error.c_str() : g_create_error.c_str(); }
+
+int64_t cb_scratch_bytes(const cb_ctx* ctx) { return ctx ? ctx->scratch_bytes : 0; }
+
+cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
+    if (!out) return fail(nullptr, CB_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (!cfg) return fail(nullptr, CB_EINVAL, "cfg is NULL");
+    const cb_config& c = *cfg;
+    if (c.n_layers < 1 || c.n_q_heads < 1 || c.n_kv_heads < 1)
+        return fail(nullptr, CB_ESHAPE, "n_layers, n_q_heads and n_kv_heads must be >= 1");
+    if (c.n_q_heads % c.n_kv_heads)
+        return fail(nullptr, CB_ESHAPE, "n_q_heads (%d) is not a multiple of n_kv_heads (%d)", c.n_q_heads,
+                    c.n_kv_heads);
+    const int G = c.n_q_heads / c.n_kv_heads;
+    if (G != 1 && G != 2 && G != 4) return fail(nullptr, CB_ESHAPE, "group size G = %d not in {1, 2, 4}", G);
+    if (c.head_dim != 64 && c.head_dim != 128)
+        return fail(nullptr, CB_ESHAPE, "head_dim %d not in {64, 128}", c.head_dim);
+    if (c.max_query_tokens < 1 || c.max_query_tokens > cbk::kMaxQueryTokens)
+        return fail(nullptr, CB_ESHAPE, "max_query_tokens %d not in [1, %d]", c.max_query_tokens,
+                    cbk::kMaxQueryTokens);
+    if (c.max_positions < 1 || c.max_positions > INT32_MAX)
+        return fail(nullptr, CB_ESHAPE, "max_positions must be in [1, 2^31)");
+    if (c.max_senders < 1 || c.max_senders > 4096)
+        return fail(nullptr, CB_ESHAPE, "max_senders %d not in [1, 4096]", c.max_senders);
+    if (!(std::isfinite(c.p) && c.p > 1.f)) return fail(nullptr, CB_EINVAL, "p must be finite and > 1");
+    if (!(std::isfinite(c.alpha) && c.alpha >= 0.f)) return fail(nullptr, CB_EINVAL, "alpha must be finite and >= 0");
+    if (!(std::isfinite(c.softmax_scale) && c.softmax_scale >= 0.f))
+        return fail(nullptr, CB_EINVAL, "softmax_scale must be finite and >= 0");
+    if (c.pool_width < 1 || c.pool_width > cbk::kMaxPoolWidth || (c.pool_width % 2) == 0)
+        return fail(nullptr, CB_EINVAL, "pool_width %d must be odd and in [1, %d]", c.pool_width,
+                    cbk::kMaxPoolWidth);
+    if (c.span_width < 1 || c.span_width > cbk::kMaxSpanWidth)
+        return fail(nullptr, CB_EINVAL, "span_width %d not in [1, %d]", c.span_width, cbk::kMaxSpanWidth);
+    if (c.n_sink < 0 || c.n_latent < 0) return fail(nullptr, CB_EINVAL, "n_sink and n_latent must be >= 0");
+
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(nullptr, CB_ECUDA, "no CUDA device: %s", cudaGetErrorString(e));
+    cb_ctx* ctx = new cb_ctx();
+    ctx->cfg = c;
+    ctx->device = dev;
+    ctx->G = G;
+    ctx->scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.f / std::sqrt((float)c.head_dim);
+    cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, dev);
+
+    const int64_t nS = (int64_t)c.n_layers * c.n_kv_heads;
+    const int64_t S = c.max_senders;
+    ctx->n_chunk1_max = (c.max_positions + cbk::kStatsChunk - 1) / cbk::kStatsChunk;
+    const int64_t rows = (int64_t)c.max_query_tokens * G;
+    ctx->keys_per_sender = (c.max_positions + c.span_width - 1) / c.span_width;
+    int64_t total = 0;
+    e = alloc(&ctx->stats, (size_t)(S * nS * ctx->n_chunk1_max * rows), &total);
+    if (e == cudaSuccess) e = alloc(&ctx->offs, (size_t)(S * nS * rows), &total);
+    if (e == cudaSuccess) e = alloc(&ctx->part, (size_t)(S * 3 * nS * c.max_positions), &total);
+    if (e == cudaSuccess) e = alloc(&ctx->span_keys, (size_t)(S * ctx->keys_per_sender), &total);
+    if (e == cudaSuccess) e = alloc(&ctx->err, 1, &total);
+    if (e == cudaSuccess) e = cudaMemset(ctx->err, 0, sizeof(uint32_t));
+    ctx->scratch_bytes = total;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        cb_destroy(ctx);
+        return fail(nullptr, CB_ENOMEM, "scratch allocation of %lld bytes failed: %s", (long long)total,
+                    cudaGetErrorString(e));
+    }
+    *out = ctx;
+    return CB_OK;
+}
+
+void cb_destroy(cb_ctx* ctx) {
+    if (!ctx) return;
+    {
+        DeviceGuard dg(ctx->device);
+        cudaDeviceSynchronize();
+        cudaFree(ctx->stats);
+        cudaFree(ctx->offs);
+        cudaFree(ctx->part);
+        cudaFree(ctx->span_keys);
+        cudaFree(ctx->err);
+    }
+    delete ctx;
+}
+
+cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query* queries, float* const* scores,
+                   void* stream) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    const cb_config& c = ctx->cfg;
+    if (n < 1 || n > c.max_senders) return fail(ctx, CB_ESHAPE, "n = %d not in [1, %d]", n, c.max_senders);
+    if (!senders || !queries || !scores) return fail(ctx, CB_EINVAL, "senders, queries or scores is NULL");
+    DeviceGuard dg(ctx->device);
+    if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
+    for (int i = 0; i < n; ++i) {
+        const cb_kv& s = senders[i];
+        const cb_query& q = queries[i];
+        if (s.T < 1 || s.T > c.max_positions)
+            return fail(ctx, CB_ESHAPE, "senders[%d].T = %lld not in [1, %lld]", i, (long long)s.T,
+                        (long long)c.max_positions);
+        if (q.m < 1 || q.m > c.max_query_tokens)
+            return fail(ctx, CB_ESHAPE, "queries[%d].m = %d not in [1, %d]", i, q.m, c.max_query_tokens);
+        if (!stride_ok(s.s_layer) || !stride_ok(s.s_head) || !stride_ok(s.s_pos) || s.s_pos < c.head_dim)
+            return fail(ctx, CB_EINVAL, "senders[%d]: strides must be positive multiples of 8 (s_pos >= d)", i);
+        if (!stride_ok(q.s_layer) || !stride_ok(q.s_tok) || !stride_ok(q.s_head) || q.s_head < c.head_dim)
+            return fail(ctx, CB_EINVAL, "queries[%d]: strides must be positive multiples of 8 (s_head >= d)", i);
+        cb_status st;
+        if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
+        if ((st = check_device_ptr(ctx, q.q, "queries.q", i))) return st;
+        if ((st = check_device_ptr(ctx, scores[i], "scores", i))) return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    const int nS = c.n_layers * c.n_kv_heads;
+    for (int b0 = 0; b0 < n; b0 += cbk::kMaxBatch) {
+        const int nb = n - b0 < cbk::kMaxBatch ? n - b0 : cbk::kMaxBatch;
+        cbk::ScoreBatch* bt = new cbk::ScoreBatch();
+        bt->n = nb;
+        bt->n_layers = c.n_layers;
+        bt->n_q_heads = c.n_q_heads;
+        bt->n_kv_heads = c.n_kv_heads;
+        bt->head_dim = c.head_dim;
+        bt->scale_log2e = ctx->scale * 1.4426950408889634f;
+        bt->p = c.p;
+        bt->alpha = c.alpha;
+        bt->pool_half = c.pool_width / 2;
+        bt->stats = ctx->stats;
+        bt->offs = ctx->offs;
+        bt->part = ctx->part;
+        int64_t so = 0, oo = 0, po = 0, b1 = 0, b2 = 0, bf = 0;
+        for (int k = 0; k < nb; ++k) {
+            const cb_kv& s = senders[b0 + k];
+            const cb_query& q = queries[b0 + k];
+            cbk::ScoreSender& d = bt->s[k];
+            d.k = static_cast<const uint16_t*>(s.k);
+            d.q = static_cast<const uint16_t*>(q.q);
+            d.scores = scores[b0 + k];
+            d.T = s.T;
+            d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
+            d.qs_l = q.s_layer; d.qs_t = q.s_tok; d.qs_h = q.s_head;
+            d.m = q.m;
+            d.n_chunk1 = (int32_t)((s.T + cbk::kStatsChunk - 1) / cbk::kStatsChunk);
+            d.n_chunk2 = (int32_t)((s.T + cbk::kAccumChunk - 1) / cbk::kAccumChunk);
+            d.stats_off = so; so += (int64_t)nS * d.n_chunk1 * q.m * ctx->G;
+            d.offs_off = oo; oo += (int64_t)nS * q.m * ctx->G;
+            d.part_off = po; po += (int64_t)3 * nS * s.T;
+            d.blk1_begin = b1; b1 += (int64_t)nS * d.n_chunk1;
+            d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
+            d.blkf_begin = bf; bf += (s.T + 239) / 240;
+        }
+        cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms);
+        delete bt;
+        if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "score launch failed: %s", cudaGetErrorString(e));
+    }
+    return CB_OK;
+}
+
+cb_status cb_select(cb_ctx* ctx, int32_t n, const float* const* scores, const int64_t* T, const int64_t* budget,
+                    int32_t* const* idx, void* stream) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    const cb_config& c = ctx->cfg;
+    if (n < 1 || n > c.max_senders) return fail(ctx, CB_ESHAPE, "n = %d not in [1, %d]", n, c.max_senders);
+    if (!scores || !T || !budget || !idx) return fail(ctx, CB_EINVAL, "scores, T, budget or idx is NULL");
+    DeviceGuard dg(ctx->device);
+    if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
+    for (int i = 0; i < n; ++i) {
+        if (T[i] < 1 || T[i] > c.max_positions)
+            return fail(ctx, CB_ESHAPE, "T[%d] = %lld not in [1, %lld]", i, (long long)T[i], (long long)c.max_positions);
+        const int64_t a = c.n_sink < T[i] ? c.n_sink : T[i];
+        const int64_t b = T[i] - c.n_latent > 0 ? T[i] - c.n_latent : 0;
+        const int64_t forced = a >= b ? T[i] : a + (T[i] - b);
+        if (budget[i] < forced || budget[i] > T[i])
+            return fail(ctx, CB_EBUDGET, "budget[%d] = %lld outside [%lld, %lld] (forced positions count toward it)",
+                        i, (long long)budget[i], (long long)forced, (long long)T[i]);
+        cb_status st;
+        if ((st = check_device_ptr(ctx, scores[i], "scores", i))) return st;
+        if ((st = check_device_ptr(ctx, idx[i], "idx", i))) return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    for (int b0 = 0; b0 < n; b0 += cbk::kMaxBatch) {
+        const int nb = n - b0 < cbk::kMaxBatch ? n - b0 : cbk::kMaxBatch;
+        cbk::SelectBatch bt;
+        std::memset(&bt, 0, sizeof bt);
+        bt.n = nb;
+        bt.n_sink = c.n_sink;
+        bt.n_latent = c.n_latent;
+        bt.span_w = c.span_width;
+        bt.err = ctx->err;
+        for (int k = 0; k < nb; ++k) {
+            bt.s[k].scores = scores[b0 + k];
+            bt.s[k].idx = idx[b0 + k];
+            bt.s[k].T = T[b0 + k];
+            bt.s[k].B = budget[b0 + k];
+            bt.s[k].span_keys = ctx->span_keys + (int64_t)k * ctx->keys_per_sender;
+        }
+        cudaError_t e = cbk::launch_select(bt, strm);
+        if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "select launch failed: %s", cudaGetErrorString(e));
+    }
+    return CB_OK;
+}
+
+cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx, const int64_t* budget,
+                     void* k_out, void* v_out, int64_t out_capacity, const int64_t* out_offset, int64_t o_layer,
+                     int64_t o_head, void* stream) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    const cb_config& c = ctx->cfg;
+    if (n < 1 || n > c.max_senders) return fail(ctx, CB_ESHAPE, "n = %d not in [1, %d]", n, c.max_senders);
+    if (!senders || !idx || !budget || !out_offset) return fail(ctx, CB_EINVAL, "senders, idx, budget or out_offset is NULL");
+    if (out_capacity < 0) return fail(ctx, CB_EINVAL, "out_capacity < 0");
+    if (!stride_ok(o_head) || !stride_ok(o_layer) || o_head < out_capacity * c.head_dim ||
+        o_layer < (int64_t)c.n_kv_heads * o_head)
+        return fail(ctx, CB_EINVAL, "output strides must be multiples of 8 and not overlap rows");
+    DeviceGuard dg(ctx->device);
+    if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
+    cb_status st;
+    if ((st = check_device_ptr(ctx, k_out, "k_out", 0))) return st;
+    if ((st = check_device_ptr(ctx, v_out, "v_out", 0))) return st;
+    for (int i = 0; i < n; ++i) {
+        const cb_kv& s = senders[i];
+        if (s.T < 1 || s.T > c.max_positions)
+            return fail(ctx, CB_ESHAPE, "senders[%d].T = %lld not in [1, %lld]", i, (long long)s.T,
+                        (long long)c.max_positions);
+        if (budget[i] < 0 || budget[i] > s.T)
+            return fail(ctx, CB_EBUDGET, "budget[%d] = %lld not in [0, T]", i, (long long)budget[i]);
+        if (out_offset[i] < 0 || out_offset[i] + budget[i] > out_capacity)
+            return fail(ctx, CB_EBUDGET, "sender %d: rows [%lld, %lld) exceed out_capacity %lld", i,
+                        (long long)out_offset[i], (long long)(out_offset[i] + budget[i]), (long long)out_capacity);
+        if ((int64_t)2 * c.n_layers * c.n_kv_heads * budget[i] * (c.head_dim / 8) >= ((int64_t)1 << 31))
+            return fail(ctx, CB_ESHAPE, "sender %d: too many rows for one launch", i);
+        if (!stride_ok(s.s_layer) || !stride_ok(s.s_head) || !stride_ok(s.s_pos) || s.s_pos < c.head_dim)
+            return fail(ctx, CB_EINVAL, "senders[%d]: strides must be positive multiples of 8 (s_pos >= d)", i);
+        if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
+        if ((st = check_device_ptr(ctx, s.v, "senders.v", i))) return st;
+        if (budget[i] > 0 && (st = check_device_ptr(ctx, idx[i], "idx", i))) return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    for (int b0 = 0; b0 < n; b0 += cbk::kMaxBatch) {
+        const int nb = n - b0 < cbk::kMaxBatch ? n - b0 : cbk::kMaxBatch;
+        cbk::CompactBatch bt;
+        std::memset(&bt, 0, sizeof bt);
+        bt.n = nb;
+        bt.n_layers = c.n_layers;
+        bt.n_kv_heads = c.n_kv_heads;
+        bt.head_dim = c.head_dim;
+        bt.k_out = static_cast<uint16_t*>(k_out);
+        bt.v_out = static_cast<uint16_t*>(v_out);
+        bt.o_layer = o_layer;
+        bt.o_head = o_head;
+        bt.err = ctx->err;
+        for (int k = 0; k < nb; ++k) {
+            const cb_kv& s = senders[b0 + k];
+            cbk::CompactSender& d = bt.s[k];
+            d.k = static_cast<const uint16_t*>(s.k);
+            d.v = static_cast<const uint16_t*>(s.v);
+            d.idx = idx[b0 + k];
+            d.T = s.T;
+            d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
+            d.B = budget[b0 + k];
+            d.out_off = out_offset[b0 + k];
+        }
+        cudaError_t e = cbk::launch_compact(bt, strm, ctx->num_sms);
+        if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "compact launch failed: %s", cudaGetErrorString(e));
+    }
+    return CB_OK;
+}
+
+cb_status cb_sync_status(cb_ctx* ctx, void* stream) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    DeviceGuard dg(ctx->device);
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t word = 0;
+    cudaError_t e = cudaMemcpyAsync(&word, ctx->err, sizeof word, cudaMemcpyDeviceToHost, strm);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(strm);
+    if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "device error: %s", cudaGetErrorString(e));
+    if (word) {
+        cudaMemsetAsync(ctx->err, 0, sizeof(uint32_t), strm);
+        cudaStreamSynchronize(strm);
+        return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s)", word,
+                    (word & cbk::kErrCompactIndex) ? " compact index outside [0, T)" : "",
+                    (word & cbk::kErrSelectBudget) ? " select count mismatch" : "");
+    }
+    return CB_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,94 @@
+// Internal interface between the C-ABI layer (cb_api.cu) and the kernels.
+// Everything here is device-side or launch plumbing; no host-side validation.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace cbk {
+
+constexpr int kMaxBatch = 64;        // senders per launch (larger calls are split)
+constexpr int kStatsChunk = 256;     // positions per pass-1 block
+constexpr int kAccumChunk = 128;     // output positions per pass-2 block
+constexpr int kHalo = 8;             // extra positions each side of a pass-2 block (>= pool_width/2)
+constexpr int kMaxPoolWidth = 15;
+constexpr int kMaxSpanWidth = 256;
+constexpr int kMaxQueryTokens = 1024;
+
+// Device error word bits (set by kernels' own bounds checks).
+constexpr uint32_t kErrCompactIndex = 1u;
+constexpr uint32_t kErrSelectBudget = 2u;
+
+struct ScoreSender {
+    const uint16_t* k;        // K[l][g][t][:] at k + l*ks_l + g*ks_h + t*ks_p
+    const uint16_t* q;        // Q[l][r][h][:] at q + l*qs_l + r*qs_t + h*qs_h
+    float* scores;            // [T]
+    int64_t T;
+    int64_t ks_l, ks_h, ks_p;
+    int64_t qs_l, qs_t, qs_h;
+    int32_t m;
+    int32_t n_chunk1;         // ceil(T / kStatsChunk)
+    int32_t n_chunk2;         // ceil(T / kAccumChunk)
+    int64_t stats_off;        // float2 offset of this sender's pass-1 partials
+    int64_t offs_off;         // float offset of this sender's per-row softmax offsets
+    int64_t part_off;         // float offset of this sender's [3][nS][T] partials
+    int64_t blk1_begin;       // first pass-1 block of this sender
+    int64_t blk2_begin;       // first pass-2 block of this sender
+    int64_t blkf_begin;       // first finalize block of this sender
+};
+
+struct ScoreBatch {
+    int32_t n;
+    int32_t n_layers, n_q_heads, n_kv_heads, head_dim;
+    float scale_log2e;        // softmax_scale * log2(e)
+    float p, alpha;
+    int32_t pool_half;        // pool_width / 2
+    float2* stats;            // pass-1 partial (max, sum) in log2 domain
+    float* offs;              // per-row log2 offsets (max + log2(sum) + log2(G))
+    float* part;              // per-group U_s, N_s, D_s partials
+    ScoreSender s[kMaxBatch];
+};
+
+struct SelectSender {
+    const float* scores;
+    int32_t* idx;
+    int64_t T;
+    int64_t B;
+    float* span_keys;         // scratch [n_spans]
+};
+
+struct SelectBatch {
+    int32_t n;
+    int32_t n_sink, n_latent, span_w;
+    uint32_t* err;
+    SelectSender s[kMaxBatch];
+};
+
+struct CompactSender {
+    const uint16_t* k;
+    const uint16_t* v;
+    const int32_t* idx;
+    int64_t T;
+    int64_t ks_l, ks_h, ks_p;
+    int64_t B;
+    int64_t out_off;
+    int64_t row_begin;        // first row (of n_layers*n_kv_heads*B*2) of this sender
+};
+
+struct CompactBatch {
+    int32_t n;
+    int32_t n_layers, n_kv_heads, head_dim;
+    uint16_t* k_out;
+    uint16_t* v_out;
+    int64_t o_layer, o_head;
+    int64_t total_rows;
+    uint32_t* err;
+    CompactSender s[kMaxBatch];
+};
+
+// Launchers (return the launch error, if any).
+cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms);
+cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);
+cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms);
+
+}  // namespace cbk

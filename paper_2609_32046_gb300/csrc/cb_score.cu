@@ -1,0 +1,472 @@
+// Score kernels: CacheBack position scores (App. C.1, App. D.2).
+//
+//   pass 1  k_stats     per (sender, KV group s, 256-position chunk): row max and
+//                       sum of exp of the logits of every (query token r, head h)
+//   combine k_combine   per (sender, s): chunk partials -> one log2 offset per row
+//   pass 2  k_accum     per (sender, s, 128-position chunk + 8-position halo):
+//                       a/G = exp2(z - offset), b = sum over the group's heads,
+//                       N_s = sum_r Pool(b_r)^p, bsum = sum_r b  ->  U_s, N_s, D_s
+//   k_finalize          per (sender, 240-position tile): fixed-order sums over s,
+//                       Q = Pool(U), C = (N/D)^(1/(p-1)), S = Q * C^alpha
+//
+// Both logit passes use the bf16 tensor cores through mma.sync m16n8k16 with fp32
+// accumulation.  Rows of one m16 tile are (8 query tokens) x (2 heads of the
+// group), so every thread holds all G heads of one token and the head sum needs
+// no shuffles.  The softmax is exact: pass 1 finds each row's max and
+// normaliser over all T positions, pass 2 recomputes the logits and normalises.
+#include <cfloat>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "cb_internal.cuh"
+
+namespace cbk {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kAccumPos = kAccumChunk + 2 * kHalo;   // 144 positions held per pass-2 block
+constexpr int kBStride = kAccumPos + 8;              // row stride of the b tile in smem (floats)
+constexpr int kSlab = 64;                            // query tokens per pass-2 slab (8 warps x 8)
+constexpr int kFinOut = kThreads - 2 * kHalo;        // outputs per finalize block
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float lg2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// x^p for x >= 0 (p > 1): exact square for p = 2, exp2(p log2 x) otherwise.
+__device__ __forceinline__ float powp(float x, float p, bool p_is_2) {
+    if (p_is_2) return x * x;
+    return x > 0.f ? ex2(p * lg2(x)) : 0.f;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem));
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t r[4], const void* smem) {
+    unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(s));
+}
+
+__device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Which sender a flat block index belongs to (senders are laid out back to back).
+template <typename F>
+__device__ __forceinline__ int find_sender(int n, int64_t blk, F begin_of) {
+    int i = 0;
+    while (i + 1 < n && begin_of(i + 1) <= blk) ++i;
+    return i;
+}
+
+// Stage K rows [tbase, tbase + npos) of one (l, g) slice into smem as 16-byte
+// chunks, chunk c of row n stored at column c ^ (n & 7) (conflict-free ldmatrix).
+// Rows outside [0, T) are zero.
+template <int D>
+__device__ __forceinline__ void stage_keys(uint4* ksm, const uint16_t* kbase, int64_t ks_p, int64_t tbase,
+                                           int npos, int64_t T) {
+    constexpr int CH = D / 8;
+    for (int e = threadIdx.x; e < npos * CH; e += kThreads) {
+        const int n = e / CH, ch = e % CH;
+        uint4* dst = ksm + n * CH + (ch ^ (n & 7));
+        const int64_t t = tbase + n;
+        if (t >= 0 && t < T)
+            cp_async16(dst, kbase + t * ks_p + ch * 8);
+        else
+            *dst = make_uint4(0u, 0u, 0u, 0u);
+    }
+    cp_async_wait_all();
+    __syncthreads();
+}
+
+// A fragments of the warp's 8 query tokens x G heads (m16 tile tt holds heads 2tt, 2tt+1).
+// Rows of absent tokens or heads are zero.
+template <int D, int G>
+__device__ __forceinline__ void load_query_frags(uint32_t (&af)[(G + 1) / 2][D / 16][4], const ScoreSender& sd,
+                                                 int l, int g, int r) {
+    const int qd = threadIdx.x & 3;
+#pragma unroll
+    for (int tt = 0; tt < (G + 1) / 2; ++tt)
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int j = 2 * tt + half;
+            const bool ok = (r < sd.m) && (j < G);
+            const uint16_t* row = sd.q + (int64_t)l * sd.qs_l + (int64_t)(ok ? r : 0) * sd.qs_t +
+                                  (int64_t)(g * G + (ok ? j : 0)) * sd.qs_h;
+#pragma unroll
+            for (int ks = 0; ks < D / 16; ++ks) {
+                uint32_t lo = 0u, hi = 0u;
+                if (ok) {
+                    lo = __ldg(reinterpret_cast<const uint32_t*>(row + 16 * ks + 2 * qd));
+                    hi = __ldg(reinterpret_cast<const uint32_t*>(row + 16 * ks + 8 + 2 * qd));
+                }
+                af[tt][ks][half] = lo;
+                af[tt][ks][2 + half] = hi;
+            }
+        }
+}
+
+// Logits of the warp's 32 rows against n8 block `nb` of the staged keys, accumulated into acc.
+template <int D, int G>
+__device__ __forceinline__ void logits_block(float (&acc)[(G + 1) / 2][4], const uint32_t (&af)[(G + 1) / 2][D / 16][4],
+                                             const uint4* ksm, int nb) {
+    constexpr int CH = D / 8;
+    const int lane = threadIdx.x & 31;
+    const int n = nb * 8 + (lane & 7);
+    const int mi = lane >> 3;
+#pragma unroll
+    for (int kc = 0; kc < D / 32; ++kc) {
+        uint32_t b[4];
+        const int ch = 4 * kc + mi;
+        ldmatrix_x4(b, ksm + n * CH + (ch ^ (n & 7)));
+#pragma unroll
+        for (int tt = 0; tt < (G + 1) / 2; ++tt) {
+            mma16816(acc[tt], af[tt][2 * kc], b[0], b[1]);
+            mma16816(acc[tt], af[tt][2 * kc + 1], b[2], b[3]);
+        }
+    }
+}
+
+__device__ __forceinline__ void online_merge(float& m, float& l, float mo, float lo) {
+    const float mn = fmaxf(m, mo);
+    if (mn == -INFINITY) return;
+    const float a = (m == -INFINITY) ? 0.f : l * ex2(m - mn);
+    const float b = (mo == -INFINITY) ? 0.f : lo * ex2(mo - mn);
+    m = mn;
+    l = a + b;
+}
+
+// ---------------------------------------------------------------------------
+// pass 1: row statistics over one 256-position chunk
+// ---------------------------------------------------------------------------
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ ScoreBatch bt) {
+    constexpr int GT = (G + 1) / 2;
+    constexpr int NBS = 4;  // n8 blocks per online-softmax step
+    extern __shared__ __align__(128) uint4 ksm[];
+    const int nS = bt.n_layers * bt.n_kv_heads;
+    const int64_t blk = blockIdx.x;
+    const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blk1_begin; });
+    const ScoreSender& sd = bt.s[i];
+    const int64_t local = blk - sd.blk1_begin;
+    const int s = (int)(local / sd.n_chunk1), c = (int)(local % sd.n_chunk1);
+    const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
+    const int64_t T = sd.T, t0 = (int64_t)c * kStatsChunk;
+    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, t0, kStatsChunk, T);
+
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int qd = lane & 3, rr = lane >> 2;
+    const int R = sd.m * G;
+    const float sl2e = bt.scale_log2e;
+    for (int tb = warp; tb * 8 < sd.m; tb += kThreads / 32) {
+        const int r = tb * 8 + rr;
+        uint32_t af[GT][D / 16][4];
+        load_query_frags<D, G>(af, sd, l, g, r);
+        float mrun[GT][2], lrun[GT][2];
+#pragma unroll
+        for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) { mrun[tt][h] = -INFINITY; lrun[tt][h] = 0.f; }
+        for (int nb0 = 0; nb0 < kStatsChunk / 8; nb0 += NBS) {
+            if (t0 + nb0 * 8 >= T) break;
+            float acc[NBS][GT][4];
+#pragma unroll
+            for (int nb = 0; nb < NBS; ++nb)
+#pragma unroll
+                for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[nb][tt][e] = 0.f;
+#pragma unroll
+            for (int nb = 0; nb < NBS; ++nb) logits_block<D, G>(acc[nb], af, ksm, nb0 + nb);
+#pragma unroll
+            for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    float v[NBS * 2];
+                    float vmax = -INFINITY;
+#pragma unroll
+                    for (int nb = 0; nb < NBS; ++nb)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int64_t pos = t0 + (nb0 + nb) * 8 + 2 * qd + e;
+                            float x = acc[nb][tt][2 * h + e] * sl2e;
+                            x = pos < T ? x : -INFINITY;
+                            v[nb * 2 + e] = x;
+                            vmax = fmaxf(vmax, x);
+                        }
+                    const float mn = fmaxf(mrun[tt][h], vmax);
+                    if (mn == -INFINITY) continue;
+                    float sum = 0.f;
+#pragma unroll
+                    for (int k = 0; k < NBS * 2; ++k) sum += ex2(v[k] - mn);
+                    lrun[tt][h] = lrun[tt][h] * ex2(mrun[tt][h] - mn) + sum;
+                    mrun[tt][h] = mn;
+                }
+        }
+#pragma unroll
+        for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                for (int off = 1; off <= 2; off <<= 1) {
+                    const float mo = __shfl_xor_sync(0xffffffffu, mrun[tt][h], off);
+                    const float lo = __shfl_xor_sync(0xffffffffu, lrun[tt][h], off);
+                    online_merge(mrun[tt][h], lrun[tt][h], mo, lo);
+                }
+                const int j = 2 * tt + h;
+                if (qd == 0 && r < sd.m && j < G)
+                    bt.stats[sd.stats_off + ((int64_t)s * sd.n_chunk1 + c) * R + r * G + j] =
+                        make_float2(mrun[tt][h], lrun[tt][h]);
+            }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// combine: per-row log2 offset = max + log2(sum) + log2(G) over all chunks
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
+    const int nS = bt.n_layers * bt.n_kv_heads;
+    const int i = blockIdx.x / nS, s = blockIdx.x % nS;
+    const ScoreSender& sd = bt.s[i];
+    const int R = sd.m * G;
+    const float lg = log2f((float)G);
+    for (int row = threadIdx.x; row < R; row += kThreads) {
+        const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
+        float M = -INFINITY;
+        for (int c = 0; c < sd.n_chunk1; ++c) M = fmaxf(M, st[(int64_t)c * R].x);
+        float L = 0.f;
+        for (int c = 0; c < sd.n_chunk1; ++c) {
+            const float2 v = st[(int64_t)c * R];
+            if (v.x != -INFINITY) L += v.y * ex2(v.x - M);
+        }
+        bt.offs[sd.offs_off + (int64_t)s * R + row] = M + log2f(L) + lg;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// pass 2: normalised attention, head mean, Pool, per-group partial sums
+// ---------------------------------------------------------------------------
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ ScoreBatch bt) {
+    constexpr int GT = (G + 1) / 2;
+    constexpr int NB = kAccumPos / 8;   // 18 n8 blocks
+    constexpr int NBS = 3;              // n8 blocks per step
+    extern __shared__ __align__(128) uint4 smem_raw[];
+    uint4* ksm = smem_raw;                                                      // [144][D/8]
+    float* bsm = reinterpret_cast<float*>(smem_raw + kAccumPos * (D / 8));     // [64][kBStride]
+    float* bsum = bsm + kSlab * kBStride;                                       // [144]
+    float* nred = bsum + kAccumPos;                                             // [2][128]
+    float* offs = nred + 2 * kAccumChunk;                                       // [m*G]
+
+    const int nS = bt.n_layers * bt.n_kv_heads;
+    const int64_t blk = blockIdx.x;
+    const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blk2_begin; });
+    const ScoreSender& sd = bt.s[i];
+    const int64_t local = blk - sd.blk2_begin;
+    const int s = (int)(local / sd.n_chunk2), c = (int)(local % sd.n_chunk2);
+    const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
+    const int64_t T = sd.T, t0 = (int64_t)c * kAccumChunk, tbase = t0 - kHalo;
+    const int R = sd.m * G;
+    for (int row = threadIdx.x; row < R; row += kThreads) offs[row] = bt.offs[sd.offs_off + (int64_t)s * R + row];
+    for (int k = threadIdx.x; k < kAccumPos; k += kThreads) bsum[k] = 0.f;
+    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, tbase, kAccumPos, T);
+
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int qd = lane & 3, rr = lane >> 2;
+    const float sl2e = bt.scale_log2e;
+    const bool p2 = (bt.p == 2.f);
+    const int ph = bt.pool_half;
+    const int pp = threadIdx.x & (kAccumChunk - 1), hf = threadIdx.x >> 7;  // pool-phase roles
+    float nacc = 0.f;
+
+    for (int slab = 0; slab * kSlab < sd.m; ++slab) {
+        const int tb = slab * (kSlab / 8) + warp;
+        const int r = tb * 8 + rr;
+        float* brow = bsm + (warp * 8 + rr) * kBStride;
+        if (tb * 8 < sd.m) {
+            uint32_t af[GT][D / 16][4];
+            load_query_frags<D, G>(af, sd, l, g, r);
+            float off[GT][2];
+#pragma unroll
+            for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int j = 2 * tt + h;
+                    off[tt][h] = (r < sd.m && j < G) ? offs[r * G + j] : INFINITY;
+                }
+            for (int nb0 = 0; nb0 < NB; nb0 += NBS) {
+                float acc[NBS][GT][4];
+#pragma unroll
+                for (int nb = 0; nb < NBS; ++nb)
+#pragma unroll
+                    for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) acc[nb][tt][e] = 0.f;
+#pragma unroll
+                for (int nb = 0; nb < NBS; ++nb) logits_block<D, G>(acc[nb], af, ksm, nb0 + nb);
+#pragma unroll
+                for (int nb = 0; nb < NBS; ++nb) {
+                    const int col = (nb0 + nb) * 8 + 2 * qd;
+                    float bv[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        float sum = 0.f;
+#pragma unroll
+                        for (int tt = 0; tt < GT; ++tt)
+#pragma unroll
+                            for (int h = 0; h < 2; ++h) sum += ex2(acc[nb][tt][2 * h + e] * sl2e - off[tt][h]);
+                        const int64_t pos = tbase + col + e;
+                        bv[e] = (pos >= 0 && pos < T) ? sum : 0.f;
+                    }
+                    *reinterpret_cast<float2*>(brow + col) = make_float2(bv[0], bv[1]);
+                }
+            }
+        } else {
+            for (int k = 2 * qd; k < kAccumPos; k += 8) *reinterpret_cast<float2*>(brow + k) = make_float2(0.f, 0.f);
+        }
+        __syncthreads();
+        // N_s: sum over this slab's tokens of Pool(b_r)^p at the block's output positions
+        {
+            const int col = pp + kHalo;
+            const int rend = min(kSlab, sd.m - slab * kSlab);
+            for (int rl = hf * (kSlab / 2); rl < min(rend, (hf + 1) * (kSlab / 2)); ++rl) {
+                const float* row = bsm + rl * kBStride + col;
+                float mx = row[-ph];
+                for (int u = -ph + 1; u <= ph; ++u) mx = fmaxf(mx, row[u]);
+                nacc += powp(mx, bt.p, p2);
+            }
+            for (int k = threadIdx.x; k < kAccumPos; k += kThreads) {
+                float acc = 0.f;
+                for (int rl = 0; rl < rend; ++rl) acc += bsm[rl * kBStride + k];
+                bsum[k] += acc;
+            }
+        }
+        __syncthreads();
+    }
+    nred[hf * kAccumChunk + pp] = nacc;
+    __syncthreads();
+    if (threadIdx.x < kAccumChunk) {
+        const int64_t t = t0 + threadIdx.x;
+        if (t < T) {
+            const int col = threadIdx.x + kHalo;
+            const float inv_m = 1.f / (float)sd.m;
+            float mx = bsum[col - ph];
+            for (int u = -ph + 1; u <= ph; ++u) mx = fmaxf(mx, bsum[col + u]);
+            const float Nv = (nred[threadIdx.x] + nred[kAccumChunk + threadIdx.x]) * inv_m;
+            const float Dv = powp(mx * inv_m, bt.p, p2);
+            const float Uv = bsum[col] * inv_m / (float)bt.n_kv_heads;
+            float* part = bt.part + sd.part_off;
+            part[((int64_t)0 * nS + s) * T + t] = Uv;
+            part[((int64_t)1 * nS + s) * T + t] = Nv;
+            part[((int64_t)2 * nS + s) * T + t] = Dv;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// finalize: fixed-order sums over the groups, Pool(U), C, S
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_finalize(const __grid_constant__ ScoreBatch bt) {
+    __shared__ float us[kThreads];
+    const int nS = bt.n_layers * bt.n_kv_heads;
+    const int64_t blk = blockIdx.x;
+    const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blkf_begin; });
+    const ScoreSender& sd = bt.s[i];
+    const int64_t T = sd.T;
+    const int64_t t = (blk - sd.blkf_begin) * kFinOut - kHalo + threadIdx.x;
+    const bool inside = (t >= 0 && t < T);
+    const bool centre = inside && threadIdx.x >= kHalo && threadIdx.x < kThreads - kHalo;
+    const float* part = bt.part + sd.part_off;
+    float U = 0.f, Nv = 0.f, Dv = 0.f;
+    if (inside) {
+        const float* pu = part + t;
+#pragma unroll 8
+        for (int s = 0; s < nS; ++s) U += pu[(int64_t)s * T];
+        if (centre) {
+            const float* pn = part + (int64_t)nS * T + t;
+            const float* pd = part + (int64_t)2 * nS * T + t;
+#pragma unroll 8
+            for (int s = 0; s < nS; ++s) Nv += pn[(int64_t)s * T];
+#pragma unroll 8
+            for (int s = 0; s < nS; ++s) Dv += pd[(int64_t)s * T];
+        }
+    }
+    us[threadIdx.x] = U;
+    __syncthreads();
+    if (centre) {
+        const int ph = bt.pool_half;
+        float Q = us[threadIdx.x - ph];
+        for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[threadIdx.x + u]);
+        const float C = Dv > FLT_MIN ? powf(Nv / Dv, 1.f / (bt.p - 1.f)) : 1.f;
+        const float S = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
+        sd.scores[t] = S;
+    }
+}
+
+template <int D, int G>
+size_t accum_smem(int max_rows) {
+    return (size_t)kAccumPos * D * 2 + (size_t)kSlab * kBStride * 4 + kAccumPos * 4 + 2 * kAccumChunk * 4 +
+           (size_t)max_rows * 4;
+}
+
+template <int D, int G>
+cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
+    int64_t nblk1 = 0, nblk2 = 0, nblkf = 0;
+    int max_rows = 0;
+    const int nS = b.n_layers * b.n_kv_heads;
+    for (int i = 0; i < b.n; ++i) {
+        nblk1 += (int64_t)nS * b.s[i].n_chunk1;
+        nblk2 += (int64_t)nS * b.s[i].n_chunk2;
+        nblkf += (b.s[i].T + kFinOut - 1) / kFinOut;
+        max_rows = max_rows > b.s[i].m * G ? max_rows : b.s[i].m * G;
+    }
+    const size_t smem1 = (size_t)kStatsChunk * D * 2;
+    const size_t smem2 = accum_smem<D, G>(max_rows);
+    cudaError_t e = cudaFuncSetAttribute(k_stats<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_accum<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+    if (e != cudaSuccess) return e;
+    k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
+    k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
+    k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
+    k_finalize<<<(unsigned)nblkf, kThreads, 0, st>>>(b);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int /*num_sms*/) {
+    const int G = b.n_q_heads / b.n_kv_heads;
+    if (b.head_dim == 128) {
+        if (G == 4) return launch_dg<128, 4>(b, st);
+        if (G == 2) return launch_dg<128, 2>(b, st);
+        if (G == 1) return launch_dg<128, 1>(b, st);
+    } else if (b.head_dim == 64) {
+        if (G == 4) return launch_dg<64, 4>(b, st);
+        if (G == 2) return launch_dg<64, 2>(b, st);
+        if (G == 1) return launch_dg<64, 1>(b, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace cbk

@@ -1,0 +1,175 @@
+"""CUDA path vs the CPU oracle on sizes the oracle finishes in seconds (GPU).
+
+Shapes span several tiles and ragged tails: 256-position stats chunks,
+128-position accumulation chunks, 8-token query blocks, 64-token slabs.
+"""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_32046_gb300 as cb
+import synth
+from gpu_helpers import (assert_scores_close, check_sender, make_cb, oracle_scores, run_path)
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    # name, shape (nL, Hq, Hkv, d), T list, m, keep, extra config
+    ("tiny_spec", None, None, None, 0.25, {}),
+    ("g4_d128_ragged", (2, 32, 8, 128), [1000], 64, 0.25, {}),
+    ("g2_d64_odd_m", (3, 8, 4, 64), [777], 20, 0.30, {}),
+    ("mha_d128", (2, 4, 4, 128), [300], 3, 0.40, {}),
+    ("two_slabs", (1, 8, 2, 128), [700], 100, 0.25, {}),
+    ("below_one_tile", (2, 8, 2, 64), [47], 5, 0.9, {}),
+    ("p3_alpha1_pool5", (2, 8, 2, 64), [600], 12, 0.2, dict(p=3.0, alpha=1.0, pool_width=5)),
+    ("mean_query_attention", (2, 8, 2, 64), [600], 12, 0.2, dict(alpha=0.0)),
+    ("no_pooling", (2, 8, 2, 64), [600], 12, 0.2, dict(pool_width=1)),
+    ("per_position_spans", (2, 8, 2, 64), [600], 12, 0.2, dict(span_width=1)),
+    ("width8_spans_p1_5", (1, 8, 4, 128), [611], 9, 0.35, dict(span_width=8, p=1.5, alpha=4.0)),
+    ("fan_in_ragged", (2, 16, 4, 128), [300, 513, 129], 33, 0.25, {}),
+]
+
+
+def _workload(name, shape, Ts, m):
+    if shape is None:
+        return synth.make_workload("tiny")
+    return synth.custom_workload(synth.Shape(*shape), Ts, m, seed=zlib.crc32(name.encode()) % 1000, n_planted_spans=2)
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_parity(case):
+    name, shape, Ts, m, keep, extra = case
+    w = _workload(name, shape, Ts, m)
+    f = run_path(w, keep, **extra)
+    kw = dict(p=extra.get("p", 2.0), alpha=extra.get("alpha", 2.0), pool_w=extra.get("pool_width", 7),
+              span_w=extra.get("span_width", 16))
+    for i, s in enumerate(w.senders):
+        check_sender(f, i, s.K, s.V, w.queries[s.task], **kw)
+
+
+def test_select_on_oracle_scores_is_exact():
+    """Both sides rank the same fp32 scores in fp32: indices must be identical."""
+    o = oracle.default()
+    w = synth.custom_workload(synth.Shape(2, 8, 2, 64), [2000, 777, 65], 16, seed=5)
+    c = make_cb(w.spec.shape, 2000, 16, 3)
+    scores, Ts, Bs, idx = [], [], [], []
+    for s in w.senders:
+        S = o.score(s.K, w.queries[0])["S"].astype(np.float32)
+        scores.append(torch.from_numpy(S).cuda())
+        Ts.append(s.T)
+        Bs.append(max(cb.budget(s.T, 0.3), min(s.T, 41)))
+        idx.append(torch.empty(Bs[-1], dtype=torch.int32, device="cuda"))
+    c.select(scores, Ts, Bs, idx)
+    c.sync_status()
+    for S, B, x in zip(scores, Bs, idx):
+        want = o.select(S.cpu().numpy(), B)
+        assert x.cpu().numpy().tolist() == want.tolist()
+
+
+def test_select_ties_and_edge_budgets_exact():
+    o = oracle.default()
+    c = cb.CacheBack(1, 1, 1, 64, 1, 5000, 1)
+    rng = np.random.default_rng(3)
+    cases = [
+        np.ones(1000, np.float32),                                # all spans tie
+        np.round(rng.random(999) * 4).astype(np.float32),         # many ties, ragged last span
+        np.zeros(300, np.float32),
+        rng.random(41).astype(np.float32),                        # everything forced
+        rng.random(4096).astype(np.float32),
+    ]
+    for S in cases:
+        T = len(S)
+        forced = min(T, 41)
+        for B in sorted({forced, min(T, forced + 1), min(T, forced + 15), min(T, forced + 16), (T + forced) // 2, T}):
+            x = torch.empty(max(B, 1), dtype=torch.int32, device="cuda")
+            c.select([torch.from_numpy(S).cuda()], [T], [B], [x])
+            c.sync_status()
+            assert x[:B].cpu().numpy().tolist() == o.select(S, B).tolist(), (T, B)
+
+
+def test_strided_inputs():
+    """K/V stored position-major [T][nL][Hkv][d] and Q [m][nL][Hq][d]: strides, not copies."""
+    w = synth.custom_workload(synth.Shape(2, 8, 2, 128), [513], 16, seed=9)
+    s = w.senders[0]
+    Kt = s.K.permute(2, 0, 1, 3).contiguous().cuda()   # [T][nL][Hkv][d]
+    Vt = s.V.permute(2, 0, 1, 3).contiguous().cuda()
+    Qt = w.queries[0].permute(1, 0, 2, 3).contiguous().cuda()
+    K, V, Q = Kt.permute(1, 2, 0, 3), Vt.permute(1, 2, 0, 3), Qt.permute(1, 0, 2, 3)
+    c = make_cb(w.spec.shape, 513, 16, 1)
+    f = cb.Filter(c, [(K, V)], [Q], 0.25)
+    f.run()
+    c.sync_status()
+    check_sender(f, 0, s.K, s.V, w.queries[0])
+
+
+def test_deterministic_across_runs_and_streams():
+    w = synth.custom_workload(synth.Shape(2, 16, 4, 128), [900, 400], 24, seed=2)
+    f1 = run_path(w, 0.25)
+    side = torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        f2 = run_path(w, 0.25)
+    torch.cuda.synchronize()
+    for a, b in zip(f1.scores, f2.scores):
+        assert torch.equal(a.view(torch.int32), b.view(torch.int32))
+    assert torch.equal(f1.k_out.view(torch.int16), f2.k_out.view(torch.int16))
+
+
+def test_scores_depend_on_the_query():
+    """Sec. 5.1 ablation: an unrelated query changes the selection."""
+    w = synth.make_workload("tiny")
+    s = w.senders[0]
+    other = synth.make_query(w.spec, seed=99, task=0).cuda()
+    c = make_cb(w.spec.shape, 512, 16, 2)
+    f = cb.Filter(c, [(s.K.cuda(), s.V.cuda())] * 2, [w.queries[0].cuda(), other], 0.25)
+    f.run()
+    c.sync_status()
+    a, b = f.indices()
+    assert set(a.cpu().tolist()) != set(b.cpu().tolist())
+    planted = {j for j in s.planted_spans}
+    got = {int(t) // 16 for t in a.cpu().tolist()}
+    assert planted <= got, "planted spans missed by the matching query"
+
+
+def test_error_paths():
+    w = synth.make_workload("tiny")
+    s = w.senders[0]
+    K, V, Q = s.K.cuda(), s.V.cuda(), w.queries[0].cuda()
+    c = make_cb(w.spec.shape, 512, 16, 1)
+    S = torch.empty(512, dtype=torch.float32, device="cuda")
+    with pytest.raises(cb.CBError) as e:       # host memory is rejected, not dereferenced
+        c.score([s.K], [Q], [S])
+    assert e.value.status == cb.CB_EINVAL
+    buf = torch.zeros(K.numel() + 8, dtype=torch.bfloat16, device="cuda")
+    Kmis = buf[1:1 + K.numel()].view(K.shape)  # 2 bytes off a 16-byte boundary
+    with pytest.raises(cb.CBError) as e:
+        c.score([Kmis], [Q], [S])
+    assert e.value.status == cb.CB_EINVAL
+    with pytest.raises(cb.CBError) as e:       # T above the creation limit
+        big = torch.zeros(2, 2, 600, 64, dtype=torch.bfloat16, device="cuda")
+        c.score([big], [Q], [torch.empty(600, device="cuda")])
+    assert e.value.status == cb.CB_ESHAPE
+    c.score([K], [Q], [S])
+    idx = torch.empty(128, dtype=torch.int32, device="cuda")
+    with pytest.raises(cb.CBError) as e:       # budget below the 41 forced positions
+        c.select([S], [512], [40], [idx])
+    assert e.value.status == cb.CB_EBUDGET
+    with pytest.raises(cb.CBError) as e:       # budget above T
+        c.select([S], [512], [513], [idx])
+    assert e.value.status == cb.CB_EBUDGET
+    ko = torch.empty(2, 2, 100, 64, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(cb.CBError) as e:       # capacity overflow
+        c.compact([K], [V], [idx], [128], ko, torch.empty_like(ko), [0])
+    assert e.value.status == cb.CB_EBUDGET
+    bad = torch.full((128,), 7, dtype=torch.int32, device="cuda")
+    bad[5] = 600                                # outside [0, T): skipped by the kernel, reported
+    ko = torch.zeros(2, 2, 128, 64, dtype=torch.bfloat16, device="cuda")
+    c.compact([K], [V], [bad], [128], ko, torch.empty_like(ko), [0])
+    with pytest.raises(cb.CBError) as e:
+        c.sync_status()
+    assert e.value.status == cb.CB_EDEVICE
+    c.sync_status()                             # the error word was cleared
+    assert torch.equal(ko[:, :, 4], K[:, :, 7])
+    assert not ko[:, :, 5].any()
