@@ -25,7 +25,7 @@ class Filter:
 
     senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors
     queries: list of Q bf16 [nL][m_i][Hq][d] device tensors, one per sender (may repeat)
-    keep:    keep ratio; budgets B_i = ceil(keep * T_i)
+    keep:    keep ratio; budgets B_i = max(ceil(keep * T_i), min(T_i, n_sink + n_latent))
     The send buffer holds every sender's rows back to back: sender i at offset sum_{j<i} B_j.
     """
 
@@ -37,7 +37,10 @@ class Filter:
         self.Qs = list(queries)
         dev = device or self.Ks[0].device
         self.Ts = [int(K.shape[2]) for K in self.Ks]
-        self.budgets = [budget(T, keep) for T in self.Ts]
+        # B_i = ceil(keep * T_i), raised to the forced count when that is larger (App. C.2: the
+        # forced first and latent positions count toward B and every budget holds them)
+        forced = cb.cfg.n_sink + cb.cfg.n_latent
+        self.budgets = [max(budget(T, keep), min(T, forced)) for T in self.Ts]
         self.offsets = []
         off = 0
         for b in self.budgets:
