@@ -169,6 +169,33 @@ const char *cb_last_error(const cb_ctx *ctx);
 /* Device scratch bytes the context holds (for capacity planning). */
 int64_t cb_scratch_bytes(const cb_ctx *ctx);
 
+/*
+ * Allocation-free selection.  The paper has no counterpart: this entry point exists
+ * for callers that cannot allocate device memory (code running inside a memory pool or
+ * arena it does not own, hosts that forbid cudaMalloc after start-up, engines whose
+ * allocator is busy or not reentrant at the point of the call), which therefore cannot
+ * hold a cb_ctx.  It computes exactly what cb_select computes, with the same kernel,
+ * and takes the selection parameters directly instead of from a context.
+ *
+ * Scratch: a fixed array of 65536 span slots (256 KiB) compiled into the library, held by
+ * every GPU that loads the library until the process exits.  One call may use at most
+ * 65536 slots in total, sum_i ceil(T[i] / span_width); larger calls return CB_ESHAPE
+ * with nothing enqueued.  The call allocates nothing: no cudaMalloc, cudaFree or
+ * allocating library routine.
+ *
+ * Set-up: the first call on each device looks up the array's device address (with that
+ * device current) and caches it; make that first call before any stream capture.
+ *
+ * Sharing: every call on a device uses the same array and finds the previous call's
+ * contents in it (the kernel rewrites every slot it reads, and the call clears its status
+ * word).  Calls whose kernels may overlap on the GPU race on the array: order them on one
+ * stream or synchronise between them.  Arguments are as for cb_select; the current CUDA
+ * device is used; errors are described by cb_last_error(NULL).
+ */
+cb_status cb_select_noalloc(int32_t n, const float *const *scores, const int64_t *T,
+                            const int64_t *budget, int32_t *const *idx, int32_t n_sink,
+                            int32_t n_latent, int32_t span_width, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,7 +20,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
-            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes"]
+            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_select_noalloc"]
 
 
 class CBError(RuntimeError):
@@ -84,6 +84,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_last_error.restype = ctypes.c_char_p
     lib.cb_scratch_bytes.argtypes = [P]
     lib.cb_scratch_bytes.restype = ctypes.c_int64
+    lib.cb_select_noalloc.argtypes = [ctypes.c_int32, P, P, P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
+    lib.cb_select_noalloc.restype = ctypes.c_int
     if path is None:
         _LIB = lib
     return lib
@@ -92,6 +94,20 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
 def budget(T: int, keep: float) -> int:
     """ceil(keep * T) in double, clamped to [0, T] (App. C.2), computed by the library."""
     return int(load_library().cb_budget(int(T), float(keep)))
+
+
+def select_noalloc(scores: Sequence, Ts: Sequence[int], budgets: Sequence[int], idx: Sequence, n_sink: int = 1,
+                   n_latent: int = 40, span_width: int = 16, stream=None):
+    """cb_select_noalloc: selection without a context and without device allocation."""
+    lib = load_library()
+    n = len(scores)
+    st = lib.cb_select_noalloc(n, _ptr_array([s.data_ptr() for s in scores]),
+                               _ptr_array([int(t) for t in Ts], ctypes.c_int64),
+                               _ptr_array([int(b) for b in budgets], ctypes.c_int64),
+                               _ptr_array([x.data_ptr() for x in idx]), n_sink, n_latent, span_width,
+                               _stream_handle(stream))
+    if st != CB_OK:
+        raise CBError(st, lib.cb_last_error(None).decode())
 
 
 def _ptr_array(values, ctype=ctypes.c_void_p):

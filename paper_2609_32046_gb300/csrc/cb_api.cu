@@ -96,6 +96,11 @@ cudaError_t alloc(T** p, size_t count, int64_t* total) {
 
 }  // namespace
 
+namespace cbk {
+// Error text of entry points that take no context (read back by cb_last_error(NULL)).
+void set_context_free_error(const char* msg) { g_create_error = msg; }
+}  // namespace cbk
+
 extern "C" {
 
 void cb_config_init(cb_config* cfg) {

@@ -86,6 +86,9 @@ struct CompactBatch {
     CompactSender s[kMaxBatch];
 };
 
+// Records the message cb_last_error(NULL) returns (entry points without a context).
+void set_context_free_error(const char* msg);
+
 // Launchers (return the launch error, if any).
 cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms);
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);

@@ -17,8 +17,12 @@
 //      so indices come out in source order.
 #include <cfloat>
 #include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
 #include <cuda_runtime.h>
 
+#include "cacheback.h"
 #include "cb_internal.cuh"
 
 namespace cbk {
@@ -264,3 +268,155 @@ cudaError_t launch_select(const SelectBatch& b, cudaStream_t st) {
 }
 
 }  // namespace cbk
+
+// ---------------------------------------------------------------------------
+// Allocation-free selection.
+//
+// Some callers cannot allocate device memory at all: code that runs inside a
+// memory pool or arena it does not own, a host that forbids cudaMalloc after
+// start-up, or an engine whose allocator is busy or not reentrant at the point
+// of the call.  cb_select_noalloc serves them: it runs the same selection kernel
+// as cb_select, needs no context, and keeps its scratch (the span means and a
+// status word) in a fixed array compiled into this library instead of calling
+// cudaMalloc.  Every GPU that loads the library holds that array until the
+// process exits.
+// ---------------------------------------------------------------------------
+namespace cbk {
+namespace {
+
+constexpr int64_t kNoAllocMaxSpans = 65536;   // span means per call: 256 KiB of floats
+
+static __device__ __align__(256) float g_noalloc_scratch[kNoAllocMaxSpans + 64];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up once
+// per device, with that device current, and cached.
+cb_status noalloc_scratch(int dev, float** out, char* msg, size_t len) {
+    if (dev < 0 || dev >= kMaxDevices) {
+        snprintf(msg, len, "device ordinal %d not supported", dev);
+        return CB_EINVAL;
+    }
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) {
+            cudaGetLastError();
+            snprintf(msg, len, "cannot resolve the scratch array on device %d: %s", dev, cudaGetErrorString(e));
+            return CB_ECUDA;
+        }
+        g_noalloc_addr[dev] = static_cast<float*>(p);
+    }
+    *out = g_noalloc_addr[dev];
+    return CB_OK;
+}
+
+cb_status noalloc_check_ptr(const void* p, int dev, const char* what, int i, char* msg, size_t len) {
+    if (!p || (reinterpret_cast<uintptr_t>(p) & 15u)) {
+        snprintf(msg, len, "%s[%d] is NULL or not 16-byte aligned", what, i);
+        return CB_EINVAL;
+    }
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        snprintf(msg, len, "%s[%d]: cannot query pointer", what, i);
+        return CB_EINVAL;
+    }
+    if (a.type == cudaMemoryTypeManaged) return CB_OK;
+    if (a.type != cudaMemoryTypeDevice || a.device != dev) {
+        snprintf(msg, len, "%s[%d] is not device memory of device %d", what, i, dev);
+        return CB_EINVAL;
+    }
+    return CB_OK;
+}
+
+}  // namespace
+}  // namespace cbk
+
+extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, const int64_t* T,
+                                       const int64_t* budget, int32_t* const* idx, int32_t n_sink,
+                                       int32_t n_latent, int32_t span_width, void* stream) {
+    using namespace cbk;
+    char msg[256] = "";
+    cb_status st = CB_OK;
+    int dev = 0;
+    float* scratch = nullptr;
+    int64_t spans = 0;
+    if (n < 1 || n > 4096) {
+        snprintf(msg, sizeof msg, "n = %d not in [1, 4096]", n);
+        st = CB_ESHAPE;
+    } else if (!scores || !T || !budget || !idx) {
+        snprintf(msg, sizeof msg, "scores, T, budget or idx is NULL");
+        st = CB_EINVAL;
+    } else if (span_width < 1 || span_width > kMaxSpanWidth || n_sink < 0 || n_latent < 0) {
+        snprintf(msg, sizeof msg, "span_width must be in [1, %d]; n_sink, n_latent >= 0", kMaxSpanWidth);
+        st = CB_EINVAL;
+    } else if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        snprintf(msg, sizeof msg, "no CUDA device");
+        st = CB_ECUDA;
+    }
+    for (int i = 0; st == CB_OK && i < n; ++i) {
+        if (T[i] < 1 || T[i] > INT32_MAX) {
+            snprintf(msg, sizeof msg, "T[%d] = %lld not in [1, 2^31)", i, (long long)T[i]);
+            st = CB_ESHAPE;
+            break;
+        }
+        const int64_t a = n_sink < T[i] ? n_sink : T[i];
+        const int64_t b = T[i] - n_latent > 0 ? T[i] - n_latent : 0;
+        const int64_t forced = a >= b ? T[i] : a + (T[i] - b);
+        if (budget[i] < forced || budget[i] > T[i]) {
+            snprintf(msg, sizeof msg, "budget[%d] = %lld outside [%lld, %lld]", i, (long long)budget[i],
+                     (long long)forced, (long long)T[i]);
+            st = CB_EBUDGET;
+            break;
+        }
+        spans += (T[i] + span_width - 1) / span_width;
+        if ((st = noalloc_check_ptr(scores[i], dev, "scores", i, msg, sizeof msg))) break;
+        if ((st = noalloc_check_ptr(idx[i], dev, "idx", i, msg, sizeof msg))) break;
+    }
+    if (st == CB_OK && spans > kNoAllocMaxSpans) {
+        snprintf(msg, sizeof msg, "the call needs %lld span slots; this entry point holds at most %lld "
+                 "(use cb_select with a context for larger calls)", (long long)spans, (long long)kNoAllocMaxSpans);
+        st = CB_ESHAPE;
+    }
+    if (st == CB_OK) st = noalloc_scratch(dev, &scratch, msg, sizeof msg);
+    if (st != CB_OK) {
+        set_context_free_error(msg);
+        return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t* status_word = reinterpret_cast<uint32_t*>(scratch + kNoAllocMaxSpans);
+    // the array keeps the previous call's contents: the status word must start at zero
+    cudaError_t e = cudaMemsetAsync(status_word, 0, sizeof(uint32_t), strm);
+    for (int b0 = 0; e == cudaSuccess && b0 < n; b0 += kMaxBatch) {
+        const int nb = n - b0 < kMaxBatch ? n - b0 : kMaxBatch;
+        SelectBatch bt;
+        memset(&bt, 0, sizeof bt);
+        bt.n = nb;
+        bt.n_sink = n_sink;
+        bt.n_latent = n_latent;
+        bt.span_w = span_width;
+        bt.err = status_word;
+        int64_t off = 0;
+        for (int k = 0; k < nb; ++k) {
+            bt.s[k].scores = scores[b0 + k];
+            bt.s[k].idx = idx[b0 + k];
+            bt.s[k].T = T[b0 + k];
+            bt.s[k].B = budget[b0 + k];
+            bt.s[k].span_keys = scratch + off;
+            off += (T[b0 + k] + span_width - 1) / span_width;
+        }
+        e = launch_select(bt, strm);
+    }
+    if (e != cudaSuccess) {
+        snprintf(msg, sizeof msg, "select launch failed: %s", cudaGetErrorString(e));
+        set_context_free_error(msg);
+        return CB_ECUDA;
+    }
+    return CB_OK;
+}
