@@ -68,6 +68,9 @@ typedef struct cb_ctx cb_ctx; /* opaque; owns device scratch only */
  *   pool_width         Pool window, odd, 1..15 (7 in the paper; 1 disables pooling)
  *   span_width         span width for selection, 1..256 (16 in the paper; 1 ranks positions)
  *   n_sink, n_latent   forced positions: the first n_sink and the last n_latent (1 and 40)
+ *   score_kernel       0: automatic (tcgen05 tensor-core passes when head_dim = 128,
+ *                      pool_width <= 7 and max_query_tokens * G <= 512, else the mma.sync
+ *                      passes); 1: mma.sync passes; 2: tcgen05 passes (CB_ESHAPE if unsupported)
  */
 typedef struct {
     int32_t n_layers, n_q_heads, n_kv_heads, head_dim;
@@ -79,6 +82,7 @@ typedef struct {
     int32_t pool_width;
     int32_t span_width;
     int32_t n_sink, n_latent;
+    int32_t score_kernel;
 } cb_config;
 
 /* One sender's cache M_S (App. A): K[l][g][t][:] at k + l*s_layer + g*s_head + t*s_pos,

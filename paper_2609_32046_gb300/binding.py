@@ -36,7 +36,7 @@ class cb_config(ctypes.Structure):
                 ("max_positions", ctypes.c_int64), ("max_senders", ctypes.c_int32),
                 ("softmax_scale", ctypes.c_float), ("p", ctypes.c_float), ("alpha", ctypes.c_float),
                 ("pool_width", ctypes.c_int32), ("span_width", ctypes.c_int32),
-                ("n_sink", ctypes.c_int32), ("n_latent", ctypes.c_int32)]
+                ("n_sink", ctypes.c_int32), ("n_latent", ctypes.c_int32), ("score_kernel", ctypes.c_int32)]
 
 
 class cb_kv(ctypes.Structure):
@@ -145,7 +145,7 @@ class CacheBack:
     def __init__(self, n_layers: int, n_q_heads: int, n_kv_heads: int, head_dim: int, max_query_tokens: int,
                  max_positions: int, max_senders: int = 1, p: float = 2.0, alpha: float = 2.0,
                  pool_width: int = 7, span_width: int = 16, n_sink: int = 1, n_latent: int = 40,
-                 softmax_scale: float = 0.0, lib_path: Optional[str] = None):
+                 softmax_scale: float = 0.0, score_kernel: int = 0, lib_path: Optional[str] = None):
         self.lib = load_library(lib_path)
         cfg = cb_config()
         self.lib.cb_config_init(ctypes.byref(cfg))
@@ -153,6 +153,7 @@ class CacheBack:
         cfg.max_query_tokens, cfg.max_positions, cfg.max_senders = max_query_tokens, max_positions, max_senders
         cfg.softmax_scale, cfg.p, cfg.alpha = softmax_scale, p, alpha
         cfg.pool_width, cfg.span_width, cfg.n_sink, cfg.n_latent = pool_width, span_width, n_sink, n_latent
+        cfg.score_kernel = score_kernel
         self.cfg = cfg
         h = ctypes.c_void_p()
         st = self.lib.cb_create(ctypes.byref(cfg), ctypes.byref(h))

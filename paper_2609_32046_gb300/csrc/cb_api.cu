@@ -21,6 +21,7 @@ struct cb_ctx {
     int device = 0;
     int num_sms = 0;
     int G = 1;
+    bool use_tc = false;
     float scale = 0.f;
     int64_t n_chunk1_max = 0;
     float2* stats = nullptr;
@@ -114,6 +115,7 @@ void cb_config_init(cb_config* cfg) {
     cfg->n_sink = 1;
     cfg->n_latent = 40;
     cfg->max_senders = 1;
+    cfg->score_kernel = 0;
 }
 
 int64_t cb_budget(int64_t T, double keep) {
@@ -158,6 +160,11 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     if (c.span_width < 1 || c.span_width > cbk::kMaxSpanWidth)
         return fail(nullptr, CB_EINVAL, "span_width %d not in [1, %d]", c.span_width, cbk::kMaxSpanWidth);
     if (c.n_sink < 0 || c.n_latent < 0) return fail(nullptr, CB_EINVAL, "n_sink and n_latent must be >= 0");
+    if (c.score_kernel < 0 || c.score_kernel > 2) return fail(nullptr, CB_EINVAL, "score_kernel must be 0, 1 or 2");
+    const bool tc_ok = cbk::tc_path_supported(c.head_dim, G, c.pool_width / 2, c.max_query_tokens);
+    if (c.score_kernel == 2 && !tc_ok)
+        return fail(nullptr, CB_ESHAPE, "tcgen05 score passes need head_dim 128, pool_width <= 7 and "
+                    "max_query_tokens * G <= 512");
 
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -166,12 +173,13 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     ctx->cfg = c;
     ctx->device = dev;
     ctx->G = G;
+    ctx->use_tc = c.score_kernel == 2 || (c.score_kernel == 0 && tc_ok);
     ctx->scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.f / std::sqrt((float)c.head_dim);
     cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, dev);
 
     const int64_t nS = (int64_t)c.n_layers * c.n_kv_heads;
     const int64_t S = c.max_senders;
-    ctx->n_chunk1_max = (c.max_positions + cbk::kStatsChunk - 1) / cbk::kStatsChunk;
+    ctx->n_chunk1_max = cbk::stats_slots(c.max_positions);
     const int64_t rows = (int64_t)c.max_query_tokens * G;
     ctx->keys_per_sender = (c.max_positions + c.span_width - 1) / c.span_width;
     int64_t total = 0;
@@ -246,10 +254,12 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->p = c.p;
         bt->alpha = c.alpha;
         bt->pool_half = c.pool_width / 2;
+        bt->use_tc = ctx->use_tc ? 1 : 0;
+        bt->err = ctx->err;
         bt->stats = ctx->stats;
         bt->offs = ctx->offs;
         bt->part = ctx->part;
-        int64_t so = 0, oo = 0, po = 0, b1 = 0, b2 = 0, bf = 0;
+        int64_t so = 0, oo = 0, po = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
             const cb_query& q = queries[b0 + k];
@@ -263,12 +273,12 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.m = q.m;
             d.n_chunk1 = (int32_t)((s.T + cbk::kStatsChunk - 1) / cbk::kStatsChunk);
             d.n_chunk2 = (int32_t)((s.T + cbk::kAccumChunk - 1) / cbk::kAccumChunk);
-            d.stats_off = so; so += (int64_t)nS * d.n_chunk1 * q.m * ctx->G;
+            d.stats_off = so; so += (int64_t)nS * cbk::stats_slots(s.T) * q.m * ctx->G;
             d.offs_off = oo; oo += (int64_t)nS * q.m * ctx->G;
             d.part_off = po; po += (int64_t)3 * nS * s.T;
             d.blk1_begin = b1; b1 += (int64_t)nS * d.n_chunk1;
             d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
-            d.blkf_begin = bf; bf += (s.T + 239) / 240;
+            d.blkf_begin = 0;  // set by the score launcher
         }
         cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms);
         delete bt;
@@ -399,6 +409,10 @@ cb_status cb_sync_status(cb_ctx* ctx, void* stream) {
     if (word) {
         cudaMemsetAsync(ctx->err, 0, sizeof(uint32_t), strm);
         cudaStreamSynchronize(strm);
+        if (word & cbk::kErrTimeout)
+            return fail(ctx, CB_ETIMEOUT,
+                        "a bounded device wait gave up (code 0x%x: bits 8+ name the wait); the results are invalid",
+                        word);
         return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s)", word,
                     (word & cbk::kErrCompactIndex) ? " compact index outside [0, T)" : "",
                     (word & cbk::kErrSelectBudget) ? " select count mismatch" : "");

@@ -8,7 +8,15 @@
 namespace cbk {
 
 constexpr int kMaxBatch = 64;        // senders per launch (larger calls are split)
-constexpr int kStatsChunk = 256;     // positions per pass-1 block
+constexpr int kStatsChunk = 256;     // positions per pass-1 block (mma.sync path)
+constexpr int kStatsChunkTc = 512;   // positions per pass-1 chunk (tcgen05 path, two partials each)
+
+// Pass-1 partial slots a sender of T positions may need on either path.
+inline int64_t stats_slots(int64_t T) {
+    const int64_t a = (T + kStatsChunk - 1) / kStatsChunk;
+    const int64_t b = 2 * ((T + kStatsChunkTc - 1) / kStatsChunkTc);
+    return a > b ? a : b;
+}
 constexpr int kAccumChunk = 128;     // output positions per pass-2 block
 constexpr int kHalo = 8;             // extra positions each side of a pass-2 block (>= pool_width/2)
 constexpr int kMaxPoolWidth = 15;
@@ -18,6 +26,7 @@ constexpr int kMaxQueryTokens = 1024;
 // Device error word bits (set by kernels' own bounds checks).
 constexpr uint32_t kErrCompactIndex = 1u;
 constexpr uint32_t kErrSelectBudget = 2u;
+constexpr uint32_t kErrTimeout = 4u;       // a bounded mbarrier wait gave up
 
 struct ScoreSender {
     const uint16_t* k;        // K[l][g][t][:] at k + l*ks_l + g*ks_h + t*ks_p
@@ -43,6 +52,8 @@ struct ScoreBatch {
     float scale_log2e;        // softmax_scale * log2(e)
     float p, alpha;
     int32_t pool_half;        // pool_width / 2
+    int32_t use_tc;           // 1: tcgen05 passes, 0: mma.sync passes
+    uint32_t* err;            // device error word
     float2* stats;            // pass-1 partial (max, sum) in log2 domain
     float* offs;              // per-row log2 offsets (max + log2(sum) + log2(G))
     float* part;              // per-group U_s, N_s, D_s partials
@@ -88,6 +99,9 @@ struct CompactBatch {
 
 // Records the message cb_last_error(NULL) returns (entry points without a context).
 void set_context_free_error(const char* msg);
+
+// True when the tcgen05 score passes handle this shape.
+bool tc_path_supported(int head_dim, int G, int pool_half, int max_query_tokens);
 
 // Launchers (return the launch error, if any).
 cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms);

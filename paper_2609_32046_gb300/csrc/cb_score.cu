@@ -27,7 +27,6 @@ constexpr int kThreads = 256;
 constexpr int kAccumPos = kAccumChunk + 2 * kHalo;   // 144 positions held per pass-2 block
 constexpr int kBStride = kAccumPos + 8;              // row stride of the b tile in smem (floats)
 constexpr int kSlab = 64;                            // query tokens per pass-2 slab (8 warps x 8)
-constexpr int kFinOut = kThreads - 2 * kHalo;        // outputs per finalize block
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -386,42 +385,64 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // finalize: fixed-order sums over the groups, Pool(U), C, S
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_finalize(const __grid_constant__ ScoreBatch bt) {
-    __shared__ float us[kThreads];
+constexpr int kFinSlices = 4;                           // groups s split over 4 threads per position
+constexpr int kFinPos = 80;                             // positions per block incl. 8-position halos
+constexpr int kFinOut2 = kFinPos - 2 * kHalo;           // 64 outputs per block
+
+__global__ void __launch_bounds__(kFinPos * kFinSlices) k_finalize(const __grid_constant__ ScoreBatch bt) {
+    __shared__ float red[3][kFinSlices][kFinPos];
+    __shared__ float us[kFinPos];
     const int nS = bt.n_layers * bt.n_kv_heads;
     const int64_t blk = blockIdx.x;
     const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blkf_begin; });
     const ScoreSender& sd = bt.s[i];
     const int64_t T = sd.T;
-    const int64_t t = (blk - sd.blkf_begin) * kFinOut - kHalo + threadIdx.x;
+    const int lp = threadIdx.x % kFinPos, sl = threadIdx.x / kFinPos;
+    const int64_t t = (blk - sd.blkf_begin) * kFinOut2 - kHalo + lp;
     const bool inside = (t >= 0 && t < T);
-    const bool centre = inside && threadIdx.x >= kHalo && threadIdx.x < kThreads - kHalo;
+    const bool centre = lp >= kHalo && lp < kFinPos - kHalo;
     const float* part = bt.part + sd.part_off;
     float U = 0.f, Nv = 0.f, Dv = 0.f;
     if (inside) {
-        const float* pu = part + t;
-#pragma unroll 8
-        for (int s = 0; s < nS; ++s) U += pu[(int64_t)s * T];
+        // slice sl adds groups sl, sl + 4, ... in increasing order
+#pragma unroll 4
+        for (int s = sl; s < nS; s += kFinSlices) U += part[(int64_t)s * T + t];
         if (centre) {
-            const float* pn = part + (int64_t)nS * T + t;
-            const float* pd = part + (int64_t)2 * nS * T + t;
-#pragma unroll 8
-            for (int s = 0; s < nS; ++s) Nv += pn[(int64_t)s * T];
-#pragma unroll 8
-            for (int s = 0; s < nS; ++s) Dv += pd[(int64_t)s * T];
+#pragma unroll 4
+            for (int s = sl; s < nS; s += kFinSlices) Nv += part[((int64_t)nS + s) * T + t];
+#pragma unroll 4
+            for (int s = sl; s < nS; s += kFinSlices) Dv += part[((int64_t)2 * nS + s) * T + t];
         }
     }
-    us[threadIdx.x] = U;
+    red[0][sl][lp] = U;
+    red[1][sl][lp] = Nv;
+    red[2][sl][lp] = Dv;
     __syncthreads();
-    if (centre) {
+    if (sl == 0) {
+        U = ((red[0][0][lp] + red[0][1][lp]) + red[0][2][lp]) + red[0][3][lp];
+        Nv = ((red[1][0][lp] + red[1][1][lp]) + red[1][2][lp]) + red[1][3][lp];
+        Dv = ((red[2][0][lp] + red[2][1][lp]) + red[2][2][lp]) + red[2][3][lp];
+        us[lp] = U;
+    }
+    __syncthreads();
+    if (sl == 0 && centre && inside) {
         const int ph = bt.pool_half;
-        float Q = us[threadIdx.x - ph];
-        for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[threadIdx.x + u]);
+        float Q = us[lp - ph];
+        for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[lp + u]);
         const float C = Dv > FLT_MIN ? powf(Nv / Dv, 1.f / (bt.p - 1.f)) : 1.f;
         const float S = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
         sd.scores[t] = S;
     }
 }
+
+cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
+    const int G = b.n_q_heads / b.n_kv_heads;
+    const int nS = b.n_layers * b.n_kv_heads;
+    k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
+    return cudaGetLastError();
+}
+
+int64_t finalize_blocks(int64_t T) { return (T + kFinOut2 - 1) / kFinOut2; }
 
 template <int D, int G>
 size_t accum_smem(int max_rows) {
@@ -437,7 +458,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     for (int i = 0; i < b.n; ++i) {
         nblk1 += (int64_t)nS * b.s[i].n_chunk1;
         nblk2 += (int64_t)nS * b.s[i].n_chunk2;
-        nblkf += (b.s[i].T + kFinOut - 1) / kFinOut;
+        nblkf += finalize_blocks(b.s[i].T);
         max_rows = max_rows > b.s[i].m * G ? max_rows : b.s[i].m * G;
     }
     const size_t smem1 = (size_t)kStatsChunk * D * 2;
@@ -449,14 +470,47 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
     k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
-    k_finalize<<<(unsigned)nblkf, kThreads, 0, st>>>(b);
+    k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(b);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int /*num_sms*/) {
-    const int G = b.n_q_heads / b.n_kv_heads;
+cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_t* err,
+                            cudaError_t (*combine)(const ScoreBatch&, cudaStream_t));
+
+cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
+    const int G = b_in.n_q_heads / b_in.n_kv_heads;
+    // finalize block ranges follow this file's finalize tile
+    ScoreBatch* bp = new ScoreBatch(b_in);
+    int64_t bf = 0;
+    for (int i = 0; i < bp->n; ++i) {
+        bp->s[i].blkf_begin = bf;
+        bf += finalize_blocks(bp->s[i].T);
+    }
+    const ScoreBatch& b = *bp;
+    struct Free { ScoreBatch* p; ~Free() { delete p; } } guard{bp};
+    if (b.use_tc) {
+        ScoreBatch* w = new ScoreBatch(b);
+        cudaError_t e = launch_score_tc(*w, st, num_sms, b.err, launch_combine);
+        if (e == cudaErrorNotSupported) {
+            // the driver rejected a tensor map for these strides: use the mma.sync passes
+            delete w;
+            ScoreBatch* v = new ScoreBatch(b);
+            v->use_tc = 0;
+            e = launch_score(*v, st, num_sms);
+            delete v;
+            return e;
+        }
+        if (e == cudaSuccess) {
+            int64_t nblkf = 0;
+            for (int i = 0; i < w->n; ++i) nblkf += finalize_blocks(w->s[i].T);
+            k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(*w);
+            e = cudaGetLastError();
+        }
+        delete w;
+        return e;
+    }
     if (b.head_dim == 128) {
         if (G == 4) return launch_dg<128, 4>(b, st);
         if (G == 2) return launch_dg<128, 2>(b, st);

@@ -1,0 +1,773 @@
+// Score passes on the 5th-generation tensor cores (tcgen05 + TMEM + TMA), sm_103a.
+//
+// Both passes contract the receiver query Q_s = [(r, h) rows x d] of one KV group
+// s = (l, g) with that group's keys K_s = [positions x d] (App. C.1: a_{l,h,r,t} is the
+// softmax over t of scale * <q, k>).  Operands are K-major bf16 tiles staged by TMA
+// with the 128-byte swizzle; one thread issues tcgen05.mma (fp32 accumulation in
+// TMEM); eight epilogue warps read TMEM with tcgen05.ld.
+//
+//   k_stats_tc  pass 1, D = Q_s K_tile^T: TMEM lane = row (r, h), column = position.
+//               Each epilogue thread owns one row and keeps its running max and
+//               sum of exp2 over the positions of a 512-position chunk.
+//   k_accum_tc  pass 2, D = K_tile Q_s^T: TMEM lane = position, column = row (r, h).
+//               Each thread owns one position: exp2(z - offset) (offset = row max +
+//               log2 of the row sum + log2 G, so the value is a / G), the head mean b
+//               and the sum over tokens stay in registers; Pool over positions runs
+//               across lanes with shuffles plus a shared-memory halo between warps.
+//               A tile is 128 positions starting 3 before its 122 output positions.
+//
+// Warp roles (320 threads, one CTA per SM, persistent over a contiguous range of
+// work units): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-9
+// epilogue (two groups of four; warp w reads TMEM lanes 32*(w%4)..+31, the two
+// groups split the columns).  K tiles flow through a ring of smem stages; TMEM
+// holds two 256-column accumulator buffers.  Every mbarrier wait is bounded (1 s);
+// on a timeout the kernel records kErrTimeout, drains its copies and MMAs, frees
+// TMEM and returns.
+#include <cfloat>
+#include <cstdint>
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <mutex>
+#include <vector>
+
+#include "cb_internal.cuh"
+#include "cb_sm100.cuh"
+
+namespace cbk {
+namespace {
+using namespace sm100;
+
+constexpr int kWarpsTc = 10;
+constexpr int kThreadsTc = kWarpsTc * 32;
+constexpr int kMaxStages = 4;
+constexpr int kTileRows = 128;          // K rows per tile
+constexpr int kTileBytes = kTileRows * 256;   // d = 128: two 64-column swizzled blocks
+constexpr int kChunk1 = kStatsChunkTc;  // pass-1 positions per chunk
+constexpr int kMargin = 3;              // pass-2 lanes before/after the output positions
+constexpr int kOutW = 32 - 2 * kMargin;          // 26 output positions per pass-2 warp
+constexpr int kOut2 = 4 * kOutW;                 // 104 output positions per pass-2 tile
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kWaitNs = 1000000000ull;      // 1 s per wait
+constexpr int kMaxTcSenders = 32;
+
+struct TcSender {
+    CUtensorMap kmap;     // 4D {d, T, Hkv, nL}, box {64, 128, 1, 1}
+    CUtensorMap kmap32;   // same tensor, box {64, 32, 1, 1}
+    CUtensorMap qmap;     // 4D {d, Hq, m, nL}, box {64, G, qbox_tok, 1}
+    float2* stats;        // this sender's pass-1 partials [nS][n_chunk1][R]
+    const float* offs;    // this sender's per-row offsets [nS][R]
+    float* part;          // this sender's partials [3][nS][T]
+    int64_t T;
+    int32_t m, R, R_pad;
+    int32_t n_chunk1, n_tile2;
+    int32_t qbox_tok, n_qbox;
+    int64_t unit1_begin, unit2_begin;
+};
+
+struct TcBatch {
+    int32_t n;
+    int32_t nL, Hq, Hkv, G;
+    int32_t stages, rpad_max;
+    float sl2e, p;
+    int32_t p_is_2, ph;
+    int64_t units1, units2;
+    uint32_t* err;
+    TcSender s[kMaxTcSenders];
+};
+
+struct Ctl {
+    uint64_t k_full[kMaxStages], k_empty[kMaxStages];
+    uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns; group g owns 2g and 2g + 1
+    uint64_t q_full, q_empty, drain;
+    uint32_t tmem_base;
+    int abort;
+};
+
+__device__ __forceinline__ uint64_t now_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait: true when the phase completed, false on abort (set by anyone) or timeout.
+// `tag` names the wait in the device error word (bit 8 + tag) when it times out.
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Ctl* ctl, uint32_t* err, int tag) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = now_ns();
+    for (uint32_t i = 1; i < (1u << 30); ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63) == 0) {
+            if (*reinterpret_cast<volatile int*>(&ctl->abort)) return false;
+            if (now_ns() - t0 > kWaitNs) {
+                *reinterpret_cast<volatile int*>(&ctl->abort) = 1;
+                atomicOr(err, kErrTimeout | (1u << (8 + tag)));
+                return false;
+            }
+        }
+    }
+    *reinterpret_cast<volatile int*>(&ctl->abort) = 1;
+    atomicOr(err, kErrTimeout);
+    return false;
+}
+
+// Wait used only on the way out (drain): bounded, ignores the abort flag.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+    const uint64_t t0 = now_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (now_ns() - t0 > kWaitNs) return;
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+    return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+struct Unit {
+    int i, s, c;   // sender, group, chunk (pass 1) or tile (pass 2)
+};
+
+__device__ __forceinline__ Unit decode1(const TcBatch& bt, int64_t u) {
+    int i = 0;
+    while (i + 1 < bt.n && bt.s[i + 1].unit1_begin <= u) ++i;
+    const int64_t local = u - bt.s[i].unit1_begin;
+    const int nch = bt.s[i].n_chunk1 / 2;   // n_chunk1 counts (chunk, group) partial slots
+    return Unit{i, (int)(local / nch), (int)(local % nch)};
+}
+
+__device__ __forceinline__ Unit decode2(const TcBatch& bt, int64_t u) {
+    int i = 0;
+    while (i + 1 < bt.n && bt.s[i + 1].unit2_begin <= u) ++i;
+    const int64_t local = u - bt.s[i].unit2_begin;
+    return Unit{i, (int)(local / bt.s[i].n_tile2), (int)(local % bt.s[i].n_tile2)};
+}
+
+// Contiguous share of `total` units for this CTA.
+__device__ __forceinline__ void my_range(int64_t total, int64_t* b, int64_t* e) {
+    *b = total * blockIdx.x / gridDim.x;
+    *e = total * (blockIdx.x + 1) / gridDim.x;
+}
+
+// Shared memory: [Q: 2 blocks x rpad x 128 B][K ring: stages x 32 KB][Ctl][epilogue scratch]
+struct Smem {
+    uint8_t* q;
+    uint8_t* k;
+    Ctl* ctl;
+    float* epi;
+};
+
+__device__ __forceinline__ Smem carve(uint8_t* raw, const TcBatch& bt) {
+    Smem sm;
+    uint8_t* base = align1024(raw);
+    sm.q = base;
+    sm.k = base + (size_t)2 * bt.rpad_max * 128;
+    sm.ctl = reinterpret_cast<Ctl*>(sm.k + (size_t)bt.stages * kTileBytes);
+    sm.epi = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sm.ctl) + 256);
+    return sm;
+}
+
+__device__ __forceinline__ void init_ctl(Ctl* ctl, int stages) {
+    for (int k = 0; k < stages; ++k) {
+        mbar_init(&ctl->k_full[k], 1);
+        mbar_init(&ctl->k_empty[k], 1);
+    }
+    for (int b = 0; b < 4; ++b) {
+        mbar_init(&ctl->t_full[b], 1);
+        mbar_init(&ctl->t_empty[b], 4);   // the four warps of the group that owns the tile
+    }
+    mbar_init(&ctl->q_full, 1);
+    mbar_init(&ctl->q_empty, 1);
+    mbar_init(&ctl->drain, 1);
+    ctl->abort = 0;
+    fence_barrier_init();
+}
+
+// Producer: Q of group s (all rows, both column blocks) into the Q region.
+__device__ __forceinline__ void load_q(const TcBatch& bt, const TcSender& sd, const Smem& sm, int l, int g) {
+    const uint32_t bytes = (uint32_t)sd.R_pad * 256u;
+    mbar_arrive_expect_tx(&sm.ctl->q_full, bytes);
+    for (int kb = 0; kb < 2; ++kb)
+        for (int b = 0; b < sd.n_qbox; ++b)
+            tma_load_4d(sm.q + (size_t)kb * bt.rpad_max * 128 + (size_t)b * sd.qbox_tok * bt.G * 128, &sd.qmap,
+                        &sm.ctl->q_full, 64 * kb, g * bt.G, b * sd.qbox_tok, l);
+}
+
+__device__ __forceinline__ void load_k(const TcSender& sd, const Smem& sm, int stage, int l, int g, int32_t t_start) {
+    uint8_t* dst = sm.k + (size_t)stage * kTileBytes;
+    mbar_arrive_expect_tx(&sm.ctl->k_full[stage], kTileBytes);
+    tma_load_4d(dst, &sd.kmap, &sm.ctl->k_full[stage], 0, t_start, g, l);
+    tma_load_4d(dst + kTileBytes / 2, &sd.kmap, &sm.ctl->k_full[stage], 64, t_start, g, l);
+}
+
+// One K = 128 contraction (8 UMMA K-steps).  a_base / b_base: first column block of each
+// operand (rows of 128 B); the second column block sits `a_blk` / `b_blk` bytes later.
+__device__ __forceinline__ void mma_k128(uint32_t d_tmem, uint32_t a_base, uint32_t a_blk, uint32_t b_base,
+                                        uint32_t b_blk, uint32_t idesc) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const uint32_t off = (uint32_t)(k & 3) * 32u;
+        const uint64_t ad = smem_desc_sw128(a_base + (k >> 2) * a_blk + off);
+        const uint64_t bd = smem_desc_sw128(b_base + (k >> 2) * b_blk + off);
+        umma_bf16(d_tmem, ad, bd, idesc, k > 0 ? 1u : 0u);
+    }
+}
+
+__device__ __forceinline__ void online_merge(float& m, float& l, float mo, float lo) {
+    const float mn = fmaxf(m, mo);
+    if (mn == -INFINITY) return;
+    const float a = (m == -INFINITY) ? 0.f : l * ex2(m - mn);
+    const float b = (mo == -INFINITY) ? 0.f : lo * ex2(mo - mn);
+    m = mn;
+    l = a + b;
+}
+
+// ===========================================================================
+// pass 1
+// ===========================================================================
+// Epilogue: the two groups of four warps take alternate K tiles (tile index within the
+// chunk, even -> group 0).  Thread = TMEM lane = row 128 h + lane of every half h; it keeps
+// the running max and sum of exp2 of its rows over its group's tiles of the chunk and writes
+// them as partial (chunk, group); the combine kernel merges all partials of a group s.
+__global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constant__ TcBatch bt) {
+    extern __shared__ uint8_t smem_raw[];
+    const Smem sm = carve(smem_raw, bt);
+    Ctl* ctl = sm.ctl;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages);
+    if (warp == 1) {
+        tmem_alloc(&ctl->tmem_base, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+    int64_t ub, ue;
+    my_range(bt.units1, &ub, &ue);
+    const int stages = bt.stages;
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (elect_one()) {
+            int64_t kt = 0, qn = 0;
+            int prev = -1;
+            bool ok = true;
+            for (int64_t u = ub; u < ue && ok; ++u) {
+                const Unit un = decode1(bt, u);
+                const TcSender& sd = bt.s[un.i];
+                const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
+                const int key = un.i * 65536 + un.s;
+                if (key != prev) {
+                    if (!(ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 0))) break;
+                    load_q(bt, sd, sm, l, g);
+                    ++qn;
+                    prev = key;
+                }
+                const int64_t c0 = (int64_t)un.c * kChunk1;
+                const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
+                for (int tile = 0; tile < nt; ++tile, ++kt) {
+                    const int st = (int)(kt % stages);
+                    if (!(ok = wait_bar(&ctl->k_empty[st], (uint32_t)(((kt / stages) & 1) ^ 1), ctl, bt.err, 1))) break;
+                    load_k(sd, sm, st, l, g, (int32_t)(c0 + tile * kTileRows));
+                }
+            }
+            // drain: every issued load must land before the CTA exits
+            for (int64_t k = kt - stages > 0 ? kt - stages : 0; k < kt; ++k)
+                drain_wait(&ctl->k_full[k % stages], (uint32_t)((k / stages) & 1));
+            if (qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (elect_one()) {
+            int64_t kt = 0, qn = 0, jg[2] = {0, 0};
+            int prev = -1;
+            bool ok = true;
+            for (int64_t u = ub; u < ue && ok; ++u) {
+                const Unit un = decode1(bt, u);
+                const TcSender& sd = bt.s[un.i];
+                const int key = un.i * 65536 + un.s;
+                if (key != prev) {
+                    if (prev >= 0) umma_commit(&ctl->q_empty);
+                    if (!(ok = wait_bar(&ctl->q_full, (uint32_t)(qn & 1), ctl, bt.err, 2))) break;
+                    tc_fence_after();
+                    ++qn;
+                    prev = key;
+                }
+                const int halves = sd.R_pad / 128;
+                const int64_t c0 = (int64_t)un.c * kChunk1;
+                const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
+                for (int tile = 0; tile < nt && ok; ++tile, ++kt) {
+                    const int st = (int)(kt % stages);
+                    if (!(ok = wait_bar(&ctl->k_full[st], (uint32_t)((kt / stages) & 1), ctl, bt.err, 3))) break;
+                    tc_fence_after();
+                    const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
+                    const int grp = tile & 1;     // epilogue group that owns this tile
+                    for (int h = 0; h < halves; ++h) {
+                        const int64_t j = jg[grp]++;
+                        const int buf = 2 * grp + (int)(j & 1);
+                        if (!(ok = wait_bar(&ctl->t_empty[buf], (uint32_t)(((j >> 1) & 1) ^ 1), ctl, bt.err, 4))) break;
+                        tc_fence_after();
+                        mma_k128(tmem + buf * 128, smem_u32(sm.q) + h * 128 * 128, (uint32_t)bt.rpad_max * 128,
+                                 kaddr, kTileBytes / 2, idesc_bf16_f32(128, 128));
+                        umma_commit(&ctl->t_full[buf]);
+                    }
+                    umma_commit(&ctl->k_empty[st]);
+                }
+            }
+            umma_commit(&ctl->drain);
+            drain_wait(&ctl->drain, 0);
+        }
+    } else {
+        // ---------------- epilogue: running max / sum per row ----------------
+        const int grp = (warp - 2) >> 2;         // takes the tiles whose index in the chunk has this parity
+        const int sp = warp & 3;                 // TMEM lane quarter
+        const int L = sp * 32 + lane;
+        const uint32_t lane_addr = (uint32_t)(sp * 32) << 16;
+        const float c = bt.sl2e;
+        int64_t j = 0;                           // this group's items so far
+        bool ok = true;
+        for (int64_t u = ub; u < ue && ok; ++u) {
+            const Unit un = decode1(bt, u);
+            const TcSender& sd = bt.s[un.i];
+            const int halves = sd.R_pad / 128;
+            const int hpairs = (halves + 1) / 2;
+            const int64_t c0 = (int64_t)un.c * kChunk1;
+            const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
+            float M[2][2], S[2][2];                 // [pair][half in pair], raw-logit max, sum of exp2
+#pragma unroll
+            for (int a = 0; a < 2; ++a)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) { M[a][h] = -INFINITY; S[a][h] = 0.f; }
+            for (int tile = 0; tile < nt && ok; ++tile) {
+                if ((tile & 1) != grp) continue;
+                const int64_t tpos = c0 + tile * kTileRows;
+                const int nvalid = (int)min((int64_t)kTileRows, sd.T - tpos);   // positions < T in this tile
+#pragma unroll
+                for (int hp = 0; hp < 2; ++hp) {
+                    if (hp >= hpairs) break;
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        if (2 * hp + hh >= halves) break;
+                        const int buf = 2 * grp + (int)(j & 1);
+                        if (!(ok = wait_bar(&ctl->t_full[buf], (uint32_t)((j >> 1) & 1), ctl, bt.err, 5))) break;
+                        ++j;
+                        tc_fence_after();
+                        float mh = M[hp][hh], shv = S[hp][hh];
+#pragma unroll 1
+                        for (int col = 0; col < kTileRows; col += 64) {
+                            float v0[32], v1[32];
+                            const uint32_t ta = tmem + lane_addr + buf * 128 + col;
+                            tmem_ld32(ta, v0);
+                            tmem_ld32(ta + 32, v1);
+                            tmem_wait_ld();
+                            if (col + 64 > nvalid) {
+#pragma unroll
+                                for (int j = 0; j < 32; ++j) {
+                                    v0[j] = col + j < nvalid ? v0[j] : -INFINITY;
+                                    v1[j] = col + 32 + j < nvalid ? v1[j] : -INFINITY;
+                                }
+                            }
+                            float vmax = v0[0];
+#pragma unroll
+                            for (int j = 1; j < 32; ++j) vmax = fmaxf(vmax, v0[j]);
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) vmax = fmaxf(vmax, v1[j]);
+                            const float mn = fmaxf(mh, vmax * c);   // c > 0: max of c*v is c * max v
+                            if (mn != -INFINITY) {
+                                float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+                                for (int j = 0; j < 32; ++j) {
+                                    s0 += ex2(fmaf(v0[j], c, -mn));
+                                    s1 += ex2(fmaf(v1[j], c, -mn));
+                                }
+                                shv = (mh == -INFINITY ? 0.f : shv * ex2(mh - mn)) + (s0 + s1);
+                                mh = mn;
+                            }
+                        }
+                        M[hp][hh] = mh;
+                        S[hp][hh] = shv;
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&ctl->t_empty[buf]);
+                    }
+                    if (!ok) break;
+                }
+            }
+            if (!ok) break;
+            // this group's partial statistics for the chunk (slot 2 c + grp); rows of halves
+            // it saw no tile of stay (-inf, 0)
+            float2* dst = sd.stats + ((int64_t)un.s * sd.n_chunk1 + 2 * un.c + grp) * sd.R;
+#pragma unroll
+            for (int hp = 0; hp < 2; ++hp)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int row = (2 * hp + hh) * 128 + L;
+                    if (2 * hp + hh < halves && row < sd.R) dst[row] = make_float2(M[hp][hh], S[hp][hh]);
+                }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// ===========================================================================
+// pass 2
+// ===========================================================================
+// Window max over lanes lane-PH .. lane+PH of x (valid for lanes 3..28, the output lanes).
+template <int PH>
+__device__ __forceinline__ float lane_pool(float x) {
+    if (PH == 0) return x;
+    if (PH == 1) {
+        const float a = __shfl_up_sync(0xffffffffu, x, 1);
+        const float b = __shfl_down_sync(0xffffffffu, x, 1);
+        return fmaxf(x, fmaxf(a, b));
+    }
+    if (PH == 2) {
+        const float a1 = fmaxf(x, __shfl_down_sync(0xffffffffu, x, 1));        // [l, l+1]
+        const float b1 = __shfl_up_sync(0xffffffffu, a1, 2);                   // [l-2, l-1]
+        return fmaxf(fmaxf(a1, b1), __shfl_down_sync(0xffffffffu, x, 2));      // [l-2, l+2]
+    }
+    const float a1 = fmaxf(x, __shfl_down_sync(0xffffffffu, x, 1));            // [l, l+1]
+    const float a2 = fmaxf(a1, __shfl_down_sync(0xffffffffu, a1, 2));          // [l, l+3]
+    return fmaxf(a2, __shfl_up_sync(0xffffffffu, a2, 3));                      // [l-3, l+3]
+}
+
+template <bool P2>
+__device__ __forceinline__ float pow_p(float x, float p) {
+    if (P2) return x * x;
+    return x > 0.f ? ex2(p * lg2(x)) : 0.f;
+}
+
+// Epilogue: each warp owns 32 TMEM lanes = positions t0 + 26 w - 3 + lane (w = lane quarter);
+// lanes 3..28 are its output positions, the 3 lanes on each side their Pool margin (the K
+// rows of the four quarters overlap by 6 positions).  The two groups take alternate tiles.
+template <int G, int PH, bool P2>
+__global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constant__ TcBatch bt) {
+    extern __shared__ uint8_t smem_raw[];
+    const Smem sm = carve(smem_raw, bt);
+    Ctl* ctl = sm.ctl;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages);
+    if (warp == 1) {
+        tmem_alloc(&ctl->tmem_base, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = ctl->tmem_base;
+    int64_t ub, ue;
+    my_range(bt.units2, &ub, &ue);
+    const int stages = bt.stages;
+
+    if (warp == 0) {
+        if (elect_one()) {
+            int64_t kt = 0, qn = 0;
+            int prev = -1;
+            bool ok = true;
+            for (int64_t u = ub; u < ue && ok; ++u) {
+                const Unit un = decode2(bt, u);
+                const TcSender& sd = bt.s[un.i];
+                const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
+                const int key = un.i * 65536 + un.s;
+                if (key != prev) {
+                    if (!(ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 8))) break;
+                    load_q(bt, sd, sm, l, g);
+                    ++qn;
+                    prev = key;
+                }
+                const int st = (int)(kt % stages);
+                if (!(ok = wait_bar(&ctl->k_empty[st], (uint32_t)(((kt / stages) & 1) ^ 1), ctl, bt.err, 9))) break;
+                // four 32-row boxes: quarter w holds positions t0 + 26 w - 3 .. + 31
+                uint8_t* dst = sm.k + (size_t)st * kTileBytes;
+                mbar_arrive_expect_tx(&ctl->k_full[st], kTileBytes);
+                const int32_t t0 = (int32_t)((int64_t)un.c * kOut2);
+                for (int w = 0; w < 4; ++w)
+                    for (int kb = 0; kb < 2; ++kb)
+                        tma_load_4d(dst + kb * (kTileBytes / 2) + w * 32 * 128, &sd.kmap32, &ctl->k_full[st],
+                                    64 * kb, t0 + kOutW * w - kMargin, g, l);
+                ++kt;
+            }
+            for (int64_t k = kt - stages > 0 ? kt - stages : 0; k < kt; ++k)
+                drain_wait(&ctl->k_full[k % stages], (uint32_t)((k / stages) & 1));
+            if (qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
+        }
+    } else if (warp == 1) {
+        if (elect_one()) {
+            int64_t kt = 0, qn = 0, jg[2] = {0, 0};
+            int prev = -1;
+            bool ok = true;
+            for (int64_t u = ub; u < ue && ok; ++u) {
+                const Unit un = decode2(bt, u);
+                const TcSender& sd = bt.s[un.i];
+                const int key = un.i * 65536 + un.s;
+                if (key != prev) {
+                    if (prev >= 0) umma_commit(&ctl->q_empty);
+                    if (!(ok = wait_bar(&ctl->q_full, (uint32_t)(qn & 1), ctl, bt.err, 10))) break;
+                    tc_fence_after();
+                    ++qn;
+                    prev = key;
+                }
+                const int st = (int)(kt % stages);
+                if (!(ok = wait_bar(&ctl->k_full[st], (uint32_t)((kt / stages) & 1), ctl, bt.err, 11))) break;
+                tc_fence_after();
+                const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
+                const int nch = (sd.R_pad + 255) / 256;
+                const int grp = (int)((u - ub) & 1);   // epilogue group that owns this tile
+                for (int c = 0; c < nch; ++c) {
+                    // group g owns the 256 columns of buffers 2g and 2g + 1 (barriers of buffer 2g)
+                    const int64_t j = jg[grp]++;
+                    if (!(ok = wait_bar(&ctl->t_empty[2 * grp], (uint32_t)((j & 1) ^ 1), ctl, bt.err, 12))) break;
+                    tc_fence_after();
+                    const int ncol = min(256, sd.R_pad - 256 * c);
+                    mma_k128(tmem + grp * 256, kaddr, kTileBytes / 2, smem_u32(sm.q) + c * 256 * 128,
+                             (uint32_t)bt.rpad_max * 128, idesc_bf16_f32(128, ncol));
+                    umma_commit(&ctl->t_full[2 * grp]);
+                }
+                umma_commit(&ctl->k_empty[st]);
+                ++kt;
+            }
+            umma_commit(&ctl->drain);
+            drain_wait(&ctl->drain, 0);
+        }
+    } else {
+        const int ew = warp - 2, grp = ew >> 2, sp = warp & 3;
+        const uint32_t lane_addr = (uint32_t)(sp * 32) << 16;
+        float* offs = sm.epi + ew * bt.rpad_max;       // this warp's copy of the row offsets
+        const float c = bt.sl2e;
+        int64_t j = 0;                           // this group's chunks so far
+        int prev = -1;
+        bool ok = true;
+        for (int64_t u = ub; u < ue && ok; ++u) {
+            const Unit un = decode2(bt, u);
+            const TcSender& sd = bt.s[un.i];
+            const int nch = (sd.R_pad + 255) / 256;
+            if (((u - ub) & 1) != grp) continue;
+            const int key = un.i * 65536 + un.s;
+            if (key != prev) {
+                __syncwarp();
+                for (int r = lane; r < sd.R_pad; r += 32)
+                    offs[r] = r < sd.R ? sd.offs[(int64_t)un.s * sd.R + r] : INFINITY;
+                __syncwarp();
+                prev = key;
+            }
+            const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
+            const bool valid = pos >= 0 && pos < sd.T;
+            float nacc = 0.f, bsum = 0.f;
+            for (int ci = 0; ci < nch && ok; ++ci) {
+                if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
+                ++j;
+                tc_fence_after();
+                const int ncol = min(256, sd.R_pad - 256 * ci);
+                const float* ofc = offs + 256 * ci;
+#pragma unroll 1
+                for (int col = 0; col < ncol; col += 64) {
+                    float v[2][32];
+                    const uint32_t ta = tmem + lane_addr + grp * 256 + col;
+                    tmem_ld32(ta, v[0]);
+                    tmem_ld32(ta + 32, v[1]);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int q = 0; q < 2; ++q) {
+                        const float* of = ofc + col + 32 * q;
+#pragma unroll
+                        for (int k = 0; k < 32 / G; ++k) {
+                            float b = 0.f;
+#pragma unroll
+                            for (int j = 0; j < G; ++j) b += ex2(fmaf(v[q][k * G + j], c, -of[k * G + j]));
+                            b = valid ? b : 0.f;
+                            bsum += b;
+                            const float pk = lane_pool<PH>(b);
+                            nacc += pow_p<P2>(pk, bt.p);
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
+            }
+            if (!ok) break;
+            const float inv_m = 1.f / (float)sd.m;
+            const float pb = lane_pool<PH>(bsum * inv_m);
+            if (valid && lane >= kMargin && lane < kMargin + kOutW) {
+                const int64_t nS = (int64_t)bt.nL * bt.Hkv;
+                sd.part[(0 * nS + un.s) * sd.T + pos] = bsum * inv_m / (float)bt.Hkv;
+                sd.part[(1 * nS + un.s) * sd.T + pos] = nacc * inv_m;
+                sd.part[(2 * nS + un.s) * sd.T + pos] = pow_p<P2>(pb, bt.p);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+PFN_cuTensorMapEncodeTiled_v12000 encoder() {
+    std::call_once(g_encode_once, [] {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        else
+            cudaGetLastError();
+    });
+    return g_encode;
+}
+
+bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4], const cuuint64_t strides_bytes[3],
+               const cuuint32_t box[4]) {
+    auto fn = encoder();
+    if (!fn) return false;
+    const cuuint32_t es[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides_bytes, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t smem_bytes(int rpad_max, int stages) {
+    return 1024 + (size_t)2 * rpad_max * 128 + (size_t)stages * kTileBytes + 256 + (size_t)8 * rpad_max * 4;
+}
+
+template <int G, int PH, bool P2>
+cudaError_t launch_accum(const TcBatch& tb, size_t smem, int grid, cudaStream_t st) {
+    cudaError_t e =
+        cudaFuncSetAttribute(k_accum_tc<G, PH, P2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_accum_tc<G, PH, P2><<<grid, kThreadsTc, smem, st>>>(tb);
+    return cudaGetLastError();
+}
+
+template <int G, bool P2>
+cudaError_t launch_accum_gp(const TcBatch& tb, size_t smem, int grid, cudaStream_t st) {
+    switch (tb.ph) {
+        case 0: return launch_accum<G, 0, P2>(tb, smem, grid, st);
+        case 1: return launch_accum<G, 1, P2>(tb, smem, grid, st);
+        case 2: return launch_accum<G, 2, P2>(tb, smem, grid, st);
+        case 3: return launch_accum<G, 3, P2>(tb, smem, grid, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
+template <int G>
+cudaError_t launch_accum_g(const TcBatch& tb, size_t smem, int grid, cudaStream_t st) {
+    return tb.p_is_2 ? launch_accum_gp<G, true>(tb, smem, grid, st) : launch_accum_gp<G, false>(tb, smem, grid, st);
+}
+
+}  // namespace
+
+bool tc_path_supported(int head_dim, int G, int pool_half, int max_query_tokens) {
+    return head_dim == 128 && (G == 1 || G == 2 || G == 4) && pool_half <= 3 && max_query_tokens * G <= 512;
+}
+
+// Pass 1, combine, pass 2 on the tensor cores for senders [0, b.n) of `b`; the caller
+// launches the finalize kernel.  `combine` is the shared statistics-combine launcher.
+cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_t* err,
+                            cudaError_t (*combine)(const ScoreBatch&, cudaStream_t)) {
+    const int G = b.n_q_heads / b.n_kv_heads;
+    const int nS = b.n_layers * b.n_kv_heads;
+    // Encode every tensor map first: if the driver rejects one (an unusual stride
+    // pattern), nothing has been launched and the caller uses the mma.sync passes.
+    std::vector<TcBatch*> batches;
+    auto free_all = [&] { for (TcBatch* p : batches) delete p; };
+    for (int b0 = 0; b0 < b.n; b0 += kMaxTcSenders) {
+        const int nb = b.n - b0 < kMaxTcSenders ? b.n - b0 : kMaxTcSenders;
+        TcBatch* tb = new TcBatch();
+        batches.push_back(tb);
+        tb->n = nb;
+        tb->nL = b.n_layers;
+        tb->Hq = b.n_q_heads;
+        tb->Hkv = b.n_kv_heads;
+        tb->G = G;
+        tb->sl2e = b.scale_log2e;
+        tb->p = b.p;
+        tb->p_is_2 = b.p == 2.f;
+        tb->ph = b.pool_half;
+        tb->err = err;
+        int rpad_max = 128;
+        int64_t u1 = 0, u2 = 0;
+        for (int k = 0; k < nb; ++k) {
+            const ScoreSender& s = b.s[b0 + k];
+            TcSender& d = tb->s[k];
+            d.T = s.T;
+            d.m = s.m;
+            d.R = s.m * G;
+            d.R_pad = (d.R + 127) / 128 * 128;
+            rpad_max = rpad_max > d.R_pad ? rpad_max : d.R_pad;
+            d.n_chunk1 = (int32_t)(2 * ((s.T + kChunk1 - 1) / kChunk1));   // one partial per (chunk, group)
+            d.n_tile2 = (int32_t)((s.T + kOut2 - 1) / kOut2);
+            d.stats = b.stats + s.stats_off;
+            d.offs = b.offs + s.offs_off;
+            d.part = b.part + s.part_off;
+            d.unit1_begin = u1;
+            u1 += (int64_t)nS * (d.n_chunk1 / 2);
+            d.unit2_begin = u2;
+            u2 += (int64_t)nS * d.n_tile2;
+            // Q arrives in boxes of at most 256 tokens that tile the padded rows exactly
+            // (R_pad is a multiple of 128, so 128-token boxes always divide it for G = 1)
+            const int tok_pad = d.R_pad / G;
+            d.qbox_tok = tok_pad <= 256 ? tok_pad : 128;
+            d.n_qbox = tok_pad / d.qbox_tok;
+            if (d.n_qbox * d.qbox_tok != tok_pad) {
+                free_all();
+                return cudaErrorNotSupported;
+            }
+            const cuuint64_t kd[4] = {128, (cuuint64_t)s.T, (cuuint64_t)b.n_kv_heads, (cuuint64_t)b.n_layers};
+            const cuuint64_t ks[3] = {(cuuint64_t)s.ks_p * 2, (cuuint64_t)s.ks_h * 2, (cuuint64_t)s.ks_l * 2};
+            const cuuint32_t kbox[4] = {64, kTileRows, 1, 1};
+            const cuuint64_t qd[4] = {128, (cuuint64_t)b.n_q_heads, (cuuint64_t)s.m, (cuuint64_t)b.n_layers};
+            const cuuint64_t qs[3] = {(cuuint64_t)s.qs_h * 2, (cuuint64_t)s.qs_t * 2, (cuuint64_t)s.qs_l * 2};
+            const cuuint32_t qbox[4] = {64, (cuuint32_t)G, (cuuint32_t)d.qbox_tok, 1};
+            const cuuint32_t kbox32[4] = {64, 32, 1, 1};
+            if (!encode_4d(&d.kmap, s.k, kd, ks, kbox) || !encode_4d(&d.kmap32, s.k, kd, ks, kbox32) ||
+                !encode_4d(&d.qmap, s.q, qd, qs, qbox)) {
+                free_all();
+                return cudaErrorNotSupported;
+            }
+        }
+        tb->rpad_max = rpad_max;
+        tb->stages = rpad_max > 256 ? 2 : 4;
+        tb->units1 = u1;
+        tb->units2 = u2;
+    }
+    cudaError_t e = cudaSuccess;
+    for (size_t k = 0; k < batches.size() && e == cudaSuccess; ++k) {
+        TcBatch* tb = batches[k];
+        const int b0 = (int)k * kMaxTcSenders;
+        const size_t smem = smem_bytes(tb->rpad_max, tb->stages);
+        e = cudaFuncSetAttribute(k_stats_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e == cudaSuccess) {
+            const int g1 = (int)(tb->units1 < num_sms ? tb->units1 : num_sms);
+            k_stats_tc<<<g1, kThreadsTc, smem, st>>>(*tb);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess) {
+            // combine reads this batch's chunk counts (512-position chunks)
+            ScoreBatch* sub = new ScoreBatch(b);
+            sub->n = tb->n;
+            for (int j = 0; j < tb->n; ++j) {
+                sub->s[j] = b.s[b0 + j];
+                sub->s[j].n_chunk1 = tb->s[j].n_chunk1;
+            }
+            e = combine(*sub, st);
+            delete sub;
+        }
+        if (e == cudaSuccess) {
+            const int g2 = (int)(tb->units2 < num_sms ? tb->units2 : num_sms);
+            if (G == 4) e = launch_accum_g<4>(*tb, smem, g2, st);
+            else if (G == 2) e = launch_accum_g<2>(*tb, smem, g2, st);
+            else e = launch_accum_g<1>(*tb, smem, g2, st);
+        }
+    }
+    free_all();
+    return e;
+}
+
+}  // namespace cbk

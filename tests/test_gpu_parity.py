@@ -30,6 +30,12 @@ CASES = [
     ("per_position_spans", (2, 8, 2, 64), [600], 12, 0.2, dict(span_width=1)),
     ("width8_spans_p1_5", (1, 8, 4, 128), [611], 9, 0.35, dict(span_width=8, p=1.5, alpha=4.0)),
     ("fan_in_ragged", (2, 16, 4, 128), [300, 513, 129], 33, 0.25, {}),
+    ("m128_two_chunks", (2, 32, 8, 128), [900], 128, 0.25, {}),
+    ("g2_m200", (1, 8, 4, 128), [555], 200, 0.25, {}),
+    ("g1_m300", (1, 2, 2, 128), [400], 300, 0.5, {}),
+    ("pool3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=3)),
+    ("pool5_p3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=5, p=3.0)),
+    ("tail_1_position", (1, 8, 2, 128), [123], 8, 0.5, {}),
 ]
 
 
@@ -39,11 +45,21 @@ def _workload(name, shape, Ts, m):
     return synth.custom_workload(synth.Shape(*shape), Ts, m, seed=zlib.crc32(name.encode()) % 1000, n_planted_spans=2)
 
 
+def _tc_supported(shape, m, extra):
+    if shape is None:
+        return False                      # the tiny workload has head_dim 64
+    nL, Hq, Hkv, d = shape
+    return d == 128 and extra.get("pool_width", 7) <= 7 and m * (Hq // Hkv) <= 512
+
+
+@pytest.mark.parametrize("kernel", [1, 2], ids=["mma_sync", "tcgen05"])
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-def test_parity(case):
+def test_parity(case, kernel):
     name, shape, Ts, m, keep, extra = case
+    if kernel == 2 and not _tc_supported(shape, m, extra):
+        pytest.skip("shape outside the tcgen05 score path")
     w = _workload(name, shape, Ts, m)
-    f = run_path(w, keep, **extra)
+    f = run_path(w, keep, score_kernel=kernel, **extra)
     kw = dict(p=extra.get("p", 2.0), alpha=extra.get("alpha", 2.0), pool_w=extra.get("pool_width", 7),
               span_w=extra.get("span_width", 16))
     for i, s in enumerate(w.senders):
