@@ -385,7 +385,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // finalize: fixed-order sums over the groups, Pool(U), C, S
 // ---------------------------------------------------------------------------
-constexpr int kFinSlices = 4;                           // groups s split over 4 threads per position
+constexpr int kFinSlices = 12;                          // groups s split over 12 threads per position
 constexpr int kFinPos = 80;                             // positions per block incl. 8-position halos
 constexpr int kFinOut2 = kFinPos - 2 * kHalo;           // 64 outputs per block
 
@@ -404,14 +404,18 @@ __global__ void __launch_bounds__(kFinPos * kFinSlices) k_finalize(const __grid_
     const float* part = bt.part + sd.part_off;
     float U = 0.f, Nv = 0.f, Dv = 0.f;
     if (inside) {
-        // slice sl adds groups sl, sl + 4, ... in increasing order
-#pragma unroll 4
-        for (int s = sl; s < nS; s += kFinSlices) U += part[(int64_t)s * T + t];
+        // slice sl adds groups sl, sl + 12, ... in increasing order
+        const float* pu = part + t;
+#pragma unroll 8
+        for (int s = sl; s < nS; s += kFinSlices) U += __ldcs(pu + (int64_t)s * T);
         if (centre) {
-#pragma unroll 4
-            for (int s = sl; s < nS; s += kFinSlices) Nv += part[((int64_t)nS + s) * T + t];
-#pragma unroll 4
-            for (int s = sl; s < nS; s += kFinSlices) Dv += part[((int64_t)2 * nS + s) * T + t];
+            const float* pn = part + (int64_t)nS * T + t;
+            const float* pd = part + (int64_t)2 * nS * T + t;
+#pragma unroll 8
+            for (int s = sl; s < nS; s += kFinSlices) {
+                Nv += __ldcs(pn + (int64_t)s * T);
+                Dv += __ldcs(pd + (int64_t)s * T);
+            }
         }
     }
     red[0][sl][lp] = U;
@@ -419,9 +423,15 @@ __global__ void __launch_bounds__(kFinPos * kFinSlices) k_finalize(const __grid_
     red[2][sl][lp] = Dv;
     __syncthreads();
     if (sl == 0) {
-        U = ((red[0][0][lp] + red[0][1][lp]) + red[0][2][lp]) + red[0][3][lp];
-        Nv = ((red[1][0][lp] + red[1][1][lp]) + red[1][2][lp]) + red[1][3][lp];
-        Dv = ((red[2][0][lp] + red[2][1][lp]) + red[2][2][lp]) + red[2][3][lp];
+        U = red[0][0][lp];
+        Nv = red[1][0][lp];
+        Dv = red[2][0][lp];
+#pragma unroll
+        for (int k = 1; k < kFinSlices; ++k) {   // fixed order: deterministic
+            U += red[0][k][lp];
+            Nv += red[1][k][lp];
+            Dv += red[2][k][lp];
+        }
         us[lp] = U;
     }
     __syncthreads();
