@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
-            int64_t kt = 0, qn = 0, jg[2] = {0, 0};
+            int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
             int prev = -1;
             bool ok = true;
             for (int64_t u = ub; u < ue && ok; ++u) {
@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                     const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
                     const int grp = tile & 1;     // epilogue group that owns this tile
                     for (int h = 0; h < halves; ++h) {
-                        const int64_t j = jg[grp]++;
+                        const int64_t j = grp ? jg1++ : jg0++;
                         const int buf = 2 * grp + (int)(j & 1);
                         if (!(ok = wait_bar(&ctl->t_empty[buf], (uint32_t)(((j >> 1) & 1) ^ 1), ctl, bt.err, 4))) break;
                         tc_fence_after();
@@ -361,25 +361,26 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                             tmem_wait_ld();
                             if (col + 64 > nvalid) {
 #pragma unroll
-                                for (int j = 0; j < 32; ++j) {
-                                    v0[j] = col + j < nvalid ? v0[j] : -INFINITY;
-                                    v1[j] = col + 32 + j < nvalid ? v1[j] : -INFINITY;
+                                for (int q = 0; q < 32; ++q) {
+                                    v0[q] = col + q < nvalid ? v0[q] : -INFINITY;
+                                    v1[q] = col + 32 + q < nvalid ? v1[q] : -INFINITY;
                                 }
                             }
-                            float vmax = v0[0];
-#pragma unroll
-                            for (int j = 1; j < 32; ++j) vmax = fmaxf(vmax, v0[j]);
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) vmax = fmaxf(vmax, v1[j]);
-                            const float mn = fmaxf(mh, vmax * c);   // c > 0: max of c*v is c * max v
+                            const float mn = fmaxf(mh, max_tree2(v0, v1) * c);   // c > 0: max of c*v is c * max v
                             if (mn != -INFINITY) {
-                                float s0 = 0.f, s1 = 0.f;
+                                const uint64_t cc = pack2(c, c), nm = pack2(-mn, -mn);
+                                uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-                                for (int j = 0; j < 32; ++j) {
-                                    s0 += ex2(fmaf(v0[j], c, -mn));
-                                    s1 += ex2(fmaf(v1[j], c, -mn));
+                                for (int q = 0; q < 16; ++q) {
+                                    float a0, a1, a2, a3;
+                                    unpack2(ffma2(pack2(v0[2 * q], v0[2 * q + 1]), cc, nm), a0, a1);
+                                    unpack2(ffma2(pack2(v1[2 * q], v1[2 * q + 1]), cc, nm), a2, a3);
+                                    acc[q & 1] = fadd2(acc[q & 1], pack2(ex2(a0), ex2(a1)));
+                                    acc[2 + (q & 1)] = fadd2(acc[2 + (q & 1)], pack2(ex2(a2), ex2(a3)));
                                 }
-                                shv = (mh == -INFINITY ? 0.f : shv * ex2(mh - mn)) + (s0 + s1);
+                                float x0, x1;
+                                unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
+                                shv = (mh == -INFINITY ? 0.f : shv * ex2(mh - mn)) + (x0 + x1);
                                 mh = mn;
                             }
                         }
@@ -494,7 +495,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         }
     } else if (warp == 1) {
         if (elect_one()) {
-            int64_t kt = 0, qn = 0, jg[2] = {0, 0};
+            int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
             int prev = -1;
             bool ok = true;
             for (int64_t u = ub; u < ue && ok; ++u) {
@@ -516,7 +517,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 const int grp = (int)((u - ub) & 1);   // epilogue group that owns this tile
                 for (int c = 0; c < nch; ++c) {
                     // group g owns the 256 columns of buffers 2g and 2g + 1 (barriers of buffer 2g)
-                    const int64_t j = jg[grp]++;
+                    const int64_t j = grp ? jg1++ : jg0++;
                     if (!(ok = wait_bar(&ctl->t_empty[2 * grp], (uint32_t)((j & 1) ^ 1), ctl, bt.err, 12))) break;
                     tc_fence_after();
                     const int ncol = min(256, sd.R_pad - 256 * c);
@@ -546,39 +547,71 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const int key = un.i * 65536 + un.s;
             if (key != prev) {
                 __syncwarp();
-                for (int r = lane; r < sd.R_pad; r += 32)
-                    offs[r] = r < sd.R ? sd.offs[(int64_t)un.s * sd.R + r] : INFINITY;
+                for (int r = lane; r < sd.R_pad; r += 32)   // stored negated: exp2(c z - offset) = exp2(fma(z, c, -offset))
+                    offs[r] = r < sd.R ? -sd.offs[(int64_t)un.s * sd.R + r] : -INFINITY;
                 __syncwarp();
                 prev = key;
             }
             const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
             const bool valid = pos >= 0 && pos < sd.T;
-            float nacc = 0.f, bsum = 0.f;
+            uint64_t nacc2 = 0ull, bsum2 = 0ull;   // pairs of token partial sums
             for (int ci = 0; ci < nch && ok; ++ci) {
                 if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
                 ++j;
                 tc_fence_after();
                 const int ncol = min(256, sd.R_pad - 256 * ci);
                 const float* ofc = offs + 256 * ci;
+                const bool all_valid = __all_sync(0xffffffffu, valid);
+                const uint64_t cc = pack2(c, c);
 #pragma unroll 1
                 for (int col = 0; col < ncol; col += 64) {
-                    float v[2][32];
+                    float v0[32], v1[32];
                     const uint32_t ta = tmem + lane_addr + grp * 256 + col;
-                    tmem_ld32(ta, v[0]);
-                    tmem_ld32(ta + 32, v[1]);
+                    tmem_ld32(ta, v0);
+                    tmem_ld32(ta + 32, v1);
                     tmem_wait_ld();
+                    const float4* of4 = reinterpret_cast<const float4*>(ofc + col);
+                    float e[64];
 #pragma unroll
-                    for (int q = 0; q < 2; ++q) {
-                        const float* of = ofc + col + 32 * q;
+                    for (int q = 0; q < 16; ++q) {
+                        const float4 o = of4[q];
+                        const int qb = 4 * (q & 7);
+                        const float z0 = q < 8 ? v0[qb] : v1[qb], z1 = q < 8 ? v0[qb + 1] : v1[qb + 1];
+                        const float z2 = q < 8 ? v0[qb + 2] : v1[qb + 2], z3 = q < 8 ? v0[qb + 3] : v1[qb + 3];
+                        float a0, a1, a2, a3;
+                        unpack2(ffma2(pack2(z0, z1), cc, pack2(o.x, o.y)), a0, a1);
+                        unpack2(ffma2(pack2(z2, z3), cc, pack2(o.z, o.w)), a2, a3);
+                        e[4 * q] = ex2(a0);
+                        e[4 * q + 1] = ex2(a1);
+                        e[4 * q + 2] = ex2(a2);
+                        e[4 * q + 3] = ex2(a3);
+                    }
+                    // b for the 64 / G tokens of these columns (a / G summed over the group's heads)
+                    constexpr int NT = 64 / G;
+                    float b[NT];
 #pragma unroll
-                        for (int k = 0; k < 32 / G; ++k) {
-                            float b = 0.f;
+                    for (int k = 0; k < NT; ++k) {
+                        if (G == 1) b[k] = e[k];
+                        if (G == 2) b[k] = e[2 * k] + e[2 * k + 1];
+                        if (G == 4) {
+                            float x0, x1;
+                            unpack2(fadd2(pack2(e[4 * k], e[4 * k + 1]), pack2(e[4 * k + 2], e[4 * k + 3])), x0, x1);
+                            b[k] = x0 + x1;
+                        }
+                    }
+                    if (!all_valid) {
 #pragma unroll
-                            for (int j = 0; j < G; ++j) b += ex2(fmaf(v[q][k * G + j], c, -of[k * G + j]));
-                            b = valid ? b : 0.f;
-                            bsum += b;
-                            const float pk = lane_pool<PH>(b);
-                            nacc += pow_p<P2>(pk, bt.p);
+                        for (int k = 0; k < NT; ++k) b[k] = valid ? b[k] : 0.f;
+                    }
+#pragma unroll
+                    for (int k = 0; k < NT; k += 2) {
+                        const float p0 = lane_pool<PH>(b[k]), p1 = lane_pool<PH>(b[k + 1]);
+                        bsum2 = fadd2(bsum2, pack2(b[k], b[k + 1]));
+                        if (P2) {
+                            const uint64_t pp = pack2(p0, p1);
+                            nacc2 = ffma2(pp, pp, nacc2);
+                        } else {
+                            nacc2 = fadd2(nacc2, pack2(pow_p<false>(p0, bt.p), pow_p<false>(p1, bt.p)));
                         }
                     }
                 }
@@ -587,6 +620,11 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
             }
             if (!ok) break;
+            float nacc, bsum, t0_, t1_;
+            unpack2(nacc2, t0_, t1_);
+            nacc = t0_ + t1_;
+            unpack2(bsum2, t0_, t1_);
+            bsum = t0_ + t1_;
             const float inv_m = 1.f / (float)sd.m;
             const float pb = lane_pool<PH>(bsum * inv_m);
             if (valid && lane >= kMargin && lane < kMargin + kOutW) {

@@ -184,6 +184,51 @@ __device__ __forceinline__ float lg2(float x) {
     return y;
 }
 
+// Packed fp32 pairs (Blackwell f32x2 ALU ops): two floats in one 64-bit register pair.
+__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void unpack2(uint64_t p, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(p));
+}
+
+// a * b + c on both halves
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// Max of two 32-value register arrays by a tree of 3-input max (depth 4).
+__device__ __forceinline__ float max_tree2(const float (&x)[32], const float (&y)[32]) {
+    float u[22];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) u[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
+    u[10] = fmax3(x[30], x[31], y[0]);
+#pragma unroll
+    for (int i = 0; i < 10; ++i) u[11 + i] = fmax3(y[3 * i + 1], y[3 * i + 2], y[3 * i + 3]);
+    u[21] = y[31];
+    const float w0 = fmax3(u[0], u[1], u[2]), w1 = fmax3(u[3], u[4], u[5]), w2 = fmax3(u[6], u[7], u[8]);
+    const float w3 = fmax3(u[9], u[10], u[11]), w4 = fmax3(u[12], u[13], u[14]), w5 = fmax3(u[15], u[16], u[17]);
+    const float w6 = fmax3(u[18], u[19], u[20]);
+    return fmax3(fmax3(w0, w1, w2), fmax3(w3, w4, w5), fmaxf(w6, u[21]));
+}
+
 __device__ __forceinline__ bool elect_one() {
     uint32_t pred;
     asm volatile(
