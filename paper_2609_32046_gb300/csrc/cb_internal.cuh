@@ -9,12 +9,12 @@ namespace cbk {
 
 constexpr int kMaxBatch = 64;        // senders per launch (larger calls are split)
 constexpr int kStatsChunk = 256;     // positions per pass-1 block (mma.sync path)
-constexpr int kStatsChunkTc = 512;   // positions per pass-1 chunk (tcgen05 path, two partials each)
+constexpr int kStatsChunkTc = 512;   // positions per pass-1 chunk (tcgen05 path, four partials each)
 
 // Pass-1 partial slots a sender of T positions may need on either path.
 inline int64_t stats_slots(int64_t T) {
     const int64_t a = (T + kStatsChunk - 1) / kStatsChunk;
-    const int64_t b = 2 * ((T + kStatsChunkTc - 1) / kStatsChunkTc);
+    const int64_t b = 4 * ((T + kStatsChunkTc - 1) / kStatsChunkTc);
     return a > b ? a : b;
 }
 constexpr int kAccumChunk = 128;     // output positions per pass-2 block

@@ -38,7 +38,7 @@ namespace cbk {
 namespace {
 using namespace sm100;
 
-constexpr int kWarpsTc = 10;
+constexpr int kWarpsTc = 18;                // 0 TMA, 1 MMA, 2..17 epilogue
 constexpr int kThreadsTc = kWarpsTc * 32;
 constexpr int kMaxStages = 4;
 constexpr int kTileRows = 128;          // K rows per tile
@@ -80,6 +80,7 @@ struct Ctl {
     uint64_t k_full[kMaxStages], k_empty[kMaxStages];
     uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns; group g owns 2g and 2g + 1
     uint64_t q_full, q_empty, drain;
+    uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]
     uint32_t tmem_base;
     int abort;
 };
@@ -130,7 +131,7 @@ __device__ __forceinline__ Unit decode1(const TcBatch& bt, int64_t u) {
     int i = 0;
     while (i + 1 < bt.n && bt.s[i + 1].unit1_begin <= u) ++i;
     const int64_t local = u - bt.s[i].unit1_begin;
-    const int nch = bt.s[i].n_chunk1 / 2;   // n_chunk1 counts (chunk, group) partial slots
+    const int nch = bt.s[i].n_chunk1 / 4;   // n_chunk1 counts (chunk, group, half) partial slots
     return Unit{i, (int)(local / nch), (int)(local % nch)};
 }
 
@@ -161,7 +162,7 @@ __device__ __forceinline__ Smem carve(uint8_t* raw, const TcBatch& bt) {
     sm.q = base;
     sm.k = base + (size_t)2 * bt.rpad_max * 128;
     sm.ctl = reinterpret_cast<Ctl*>(sm.k + (size_t)bt.stages * kTileBytes);
-    sm.epi = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sm.ctl) + 256);
+    sm.epi = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sm.ctl) + 512);
     return sm;
 }
 
@@ -172,11 +173,12 @@ __device__ __forceinline__ void init_ctl(Ctl* ctl, int stages) {
     }
     for (int b = 0; b < 4; ++b) {
         mbar_init(&ctl->t_full[b], 1);
-        mbar_init(&ctl->t_empty[b], 4);   // the four warps of the group that owns the tile
+        mbar_init(&ctl->t_empty[b], 8);   // the eight warps of the group that owns the tile
     }
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
     mbar_init(&ctl->drain, 1);
+    for (int k = 0; k < 16; ++k) mbar_init(&ctl->xb[k >> 3][(k >> 2) & 1][k & 3], 1);
     ctl->abort = 0;
     fence_barrier_init();
 }
@@ -200,14 +202,15 @@ __device__ __forceinline__ void load_k(const TcSender& sd, const Smem& sm, int s
 
 // One K = 128 contraction (8 UMMA K-steps).  a_base / b_base: first column block of each
 // operand (rows of 128 B); the second column block sits `a_blk` / `b_blk` bytes later.
+// The descriptors are built once; a K-step only moves the start-address field.
 __device__ __forceinline__ void mma_k128(uint32_t d_tmem, uint32_t a_base, uint32_t a_blk, uint32_t b_base,
                                         uint32_t b_blk, uint32_t idesc) {
+    const uint64_t ad0 = smem_desc_sw128(a_base), bd0 = smem_desc_sw128(b_base);
+    const uint64_t ad1 = ad0 + (a_blk >> 4), bd1 = bd0 + (b_blk >> 4);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-        const uint32_t off = (uint32_t)(k & 3) * 32u;
-        const uint64_t ad = smem_desc_sw128(a_base + (k >> 2) * a_blk + off);
-        const uint64_t bd = smem_desc_sw128(b_base + (k >> 2) * b_blk + off);
-        umma_bf16(d_tmem, ad, bd, idesc, k > 0 ? 1u : 0u);
+        const uint64_t off = (uint64_t)((k & 3) * 2);   // 32 bytes >> 4
+        umma_bf16(d_tmem, (k < 4 ? ad0 : ad1) + off, (k < 4 ? bd0 : bd1) + off, idesc, k > 0 ? 1u : 0u);
     }
 }
 
@@ -218,6 +221,45 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float mo, float
     const float b = (mo == -INFINITY) ? 0.f : lo * ex2(mo - mn);
     m = mn;
     l = a + b;
+}
+
+// One 32-column block of pass 1 for this lane's row: running offset m (log2 domain) and
+// sum of exp2(c z - m).  The first block sets m to its max; later blocks reuse m and are
+// redone with their own max only if their sum could leave fp32 range (rare).
+__device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c, uint64_t cc, float& m, float& sum) {
+    if (nvalid < 32) {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) v[q] = q < nvalid ? v[q] : -INFINITY;
+    }
+    if (m == -INFINITY) m = max_tree1(v) * c;
+    if (m == -INFINITY) return;
+    uint64_t nm = pack2(-m, -m);
+    uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+        float a0, a1;
+        unpack2(ffma2(pack2(v[2 * q], v[2 * q + 1]), cc, nm), a0, a1);
+        acc[q & 3] = fadd2(acc[q & 3], pack2(ex2(a0), ex2(a1)));
+    }
+    float x0, x1;
+    unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
+    float blk = x0 + x1;
+    if (!(blk <= 0x1p64f)) {
+        const float mn = fmaxf(m, max_tree1(v) * c);
+        nm = pack2(-mn, -mn);
+        acc[0] = acc[1] = acc[2] = acc[3] = 0ull;
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+            float a0, a1;
+            unpack2(ffma2(pack2(v[2 * q], v[2 * q + 1]), cc, nm), a0, a1);
+            acc[q & 3] = fadd2(acc[q & 3], pack2(ex2(a0), ex2(a1)));
+        }
+        unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
+        blk = x0 + x1;
+        sum *= ex2(m - mn);
+        m = mn;
+    }
+    sum += blk;
 }
 
 // ===========================================================================
@@ -318,92 +360,62 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
         }
     } else {
         // ---------------- epilogue: running max / sum per row ----------------
-        const int grp = (warp - 2) >> 2;         // takes the tiles whose index in the chunk has this parity
+        // 16 warps: quad = (warp - 2) / 4; group = quad / 2 takes the tiles whose index in the
+        // chunk has its parity, half = quad % 2 takes positions half*64 .. +64 of each tile.
+        const int quad = (warp - 2) >> 2, grp = quad >> 1, hf = quad & 1;
         const int sp = warp & 3;                 // TMEM lane quarter
         const int L = sp * 32 + lane;
         const uint32_t lane_addr = (uint32_t)(sp * 32) << 16;
         const float c = bt.sl2e;
-        int64_t j = 0;                           // this group's items so far
+        const uint64_t cc = pack2(c, c);
+        int64_t j = 0;                           // items of this group so far
         bool ok = true;
         for (int64_t u = ub; u < ue && ok; ++u) {
             const Unit un = decode1(bt, u);
             const TcSender& sd = bt.s[un.i];
             const int halves = sd.R_pad / 128;
-            const int hpairs = (halves + 1) / 2;
             const int64_t c0 = (int64_t)un.c * kChunk1;
             const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
-            float M[2][2], S[2][2];                 // [pair][half in pair], raw-logit max, sum of exp2
+            float M[4], S[4];                    // per half: offset (log2 domain) and sum of exp2(c z - offset)
 #pragma unroll
-            for (int a = 0; a < 2; ++a)
-#pragma unroll
-                for (int h = 0; h < 2; ++h) { M[a][h] = -INFINITY; S[a][h] = 0.f; }
+            for (int h = 0; h < 4; ++h) { M[h] = -INFINITY; S[h] = 0.f; }
             for (int tile = 0; tile < nt && ok; ++tile) {
                 if ((tile & 1) != grp) continue;
-                const int64_t tpos = c0 + tile * kTileRows;
-                const int nvalid = (int)min((int64_t)kTileRows, sd.T - tpos);   // positions < T in this tile
+                const int nvalid = (int)min((int64_t)kTileRows, sd.T - (c0 + tile * kTileRows)) - hf * 64;
 #pragma unroll
-                for (int hp = 0; hp < 2; ++hp) {
-                    if (hp >= hpairs) break;
+                for (int h = 0; h < 4; ++h) {
+                    if (h >= halves) break;
+                    const int buf = 2 * grp + (int)(j & 1);
+                    if (!(ok = wait_bar(&ctl->t_full[buf], (uint32_t)((j >> 1) & 1), ctl, bt.err, 5))) break;
+                    ++j;
+                    tc_fence_after();
+                    const uint32_t ta = tmem + lane_addr + buf * 128 + hf * 64;
+                    float m = M[h], sum = S[h];
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        if (2 * hp + hh >= halves) break;
-                        const int buf = 2 * grp + (int)(j & 1);
-                        if (!(ok = wait_bar(&ctl->t_full[buf], (uint32_t)((j >> 1) & 1), ctl, bt.err, 5))) break;
-                        ++j;
-                        tc_fence_after();
-                        float mh = M[hp][hh], shv = S[hp][hh];
-#pragma unroll 1
-                        for (int col = 0; col < kTileRows; col += 64) {
-                            float v0[32], v1[32];
-                            const uint32_t ta = tmem + lane_addr + buf * 128 + col;
-                            tmem_ld32(ta, v0);
-                            tmem_ld32(ta + 32, v1);
-                            tmem_wait_ld();
-                            if (col + 64 > nvalid) {
-#pragma unroll
-                                for (int q = 0; q < 32; ++q) {
-                                    v0[q] = col + q < nvalid ? v0[q] : -INFINITY;
-                                    v1[q] = col + 32 + q < nvalid ? v1[q] : -INFINITY;
-                                }
-                            }
-                            const float mn = fmaxf(mh, max_tree2(v0, v1) * c);   // c > 0: max of c*v is c * max v
-                            if (mn != -INFINITY) {
-                                const uint64_t cc = pack2(c, c), nm = pack2(-mn, -mn);
-                                uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-                                for (int q = 0; q < 16; ++q) {
-                                    float a0, a1, a2, a3;
-                                    unpack2(ffma2(pack2(v0[2 * q], v0[2 * q + 1]), cc, nm), a0, a1);
-                                    unpack2(ffma2(pack2(v1[2 * q], v1[2 * q + 1]), cc, nm), a2, a3);
-                                    acc[q & 1] = fadd2(acc[q & 1], pack2(ex2(a0), ex2(a1)));
-                                    acc[2 + (q & 1)] = fadd2(acc[2 + (q & 1)], pack2(ex2(a2), ex2(a3)));
-                                }
-                                float x0, x1;
-                                unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
-                                shv = (mh == -INFINITY ? 0.f : shv * ex2(mh - mn)) + (x0 + x1);
-                                mh = mn;
-                            }
+                    for (int half32 = 0; half32 < 2; ++half32) {
+                        float v[32];
+                        tmem_ld32(ta + 32 * half32, v);
+                        tmem_wait_ld();
+                        if (half32 == 1) {
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&ctl->t_empty[buf]);   // registers hold the rest
                         }
-                        M[hp][hh] = mh;
-                        S[hp][hh] = shv;
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&ctl->t_empty[buf]);
+                        stats_block(v, nvalid - 32 * half32, c, cc, m, sum);
                     }
-                    if (!ok) break;
+                    M[h] = m;
+                    S[h] = sum;
                 }
             }
             if (!ok) break;
-            // this group's partial statistics for the chunk (slot 2 c + grp); rows of halves
-            // it saw no tile of stay (-inf, 0)
-            float2* dst = sd.stats + ((int64_t)un.s * sd.n_chunk1 + 2 * un.c + grp) * sd.R;
+            // this warp's partial statistics for the chunk: slot 4 c + 2 grp + hf (rows of
+            // tiles it saw none of stay (-inf, 0)); the combine kernel merges all slots
+            float2* dst = sd.stats + ((int64_t)un.s * sd.n_chunk1 + 4 * un.c + 2 * grp + hf) * sd.R;
 #pragma unroll
-            for (int hp = 0; hp < 2; ++hp)
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    const int row = (2 * hp + hh) * 128 + L;
-                    if (2 * hp + hh < halves && row < sd.R) dst[row] = make_float2(M[hp][hh], S[hp][hh]);
-                }
+            for (int h = 0; h < 4; ++h) {
+                const int row = h * 128 + L;
+                if (h < halves && row < sd.R) dst[row] = make_float2(M[h], S[h]);
+            }
         }
     }
     tc_fence_before();
@@ -437,6 +449,54 @@ template <bool P2>
 __device__ __forceinline__ float pow_p(float x, float p) {
     if (P2) return x * x;
     return x > 0.f ? ex2(p * lg2(x)) : 0.f;
+}
+
+// One 32-column block of pass 2 for this lane's position: a / G = exp2(c z - offset) per
+// column, b = sum over the G heads of each token, then Pool over positions and the sums.
+template <int G, int PH, bool P2>
+__device__ __forceinline__ void accum_block(const float (&v)[32], const float* negoff, uint64_t cc, bool valid,
+                                            bool all_valid, float p, uint64_t (&nacc2)[2], uint64_t (&bsum2)[2]) {
+    const float4* of4 = reinterpret_cast<const float4*>(negoff);
+    float e[32];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const float4 o = of4[q];
+        float a0, a1, a2, a3;
+        unpack2(ffma2(pack2(v[4 * q], v[4 * q + 1]), cc, pack2(o.x, o.y)), a0, a1);
+        unpack2(ffma2(pack2(v[4 * q + 2], v[4 * q + 3]), cc, pack2(o.z, o.w)), a2, a3);
+        e[4 * q] = ex2(a0);
+        e[4 * q + 1] = ex2(a1);
+        e[4 * q + 2] = ex2(a2);
+        e[4 * q + 3] = ex2(a3);
+    }
+    constexpr int NT = 32 / G;   // tokens in these 32 columns
+    float b[NT];
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+        if (G == 1) b[k] = e[k];
+        if (G == 2) b[k] = e[2 * k] + e[2 * k + 1];
+        if (G == 4) {
+            float x0, x1;
+            unpack2(fadd2(pack2(e[4 * k], e[4 * k + 1]), pack2(e[4 * k + 2], e[4 * k + 3])), x0, x1);
+            b[k] = x0 + x1;
+        }
+    }
+    if (!all_valid) {
+#pragma unroll
+        for (int k = 0; k < NT; ++k) b[k] = valid ? b[k] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < NT; k += 2) {
+        const float p0 = lane_pool<PH>(b[k]), p1 = lane_pool<PH>(b[k + 1]);
+        const int a = (k >> 1) & 1;
+        bsum2[a] = fadd2(bsum2[a], pack2(b[k], b[k + 1]));
+        if (P2) {
+            const uint64_t pp = pack2(p0, p1);
+            nacc2[a] = ffma2(pp, pp, nacc2[a]);
+        } else {
+            nacc2[a] = fadd2(nacc2[a], pack2(pow_p<false>(p0, p), pow_p<false>(p1, p)));
+        }
+    }
 }
 
 // Epilogue: each warp owns 32 TMEM lanes = positions t0 + 26 w - 3 + lane (w = lane quarter);
@@ -532,11 +592,15 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             drain_wait(&ctl->drain, 0);
         }
     } else {
-        const int ew = warp - 2, grp = ew >> 2, sp = warp & 3;
+        // 16 warps: quad = (warp - 2) / 4; group = quad / 2 takes alternate tiles, half = quad % 2
+        // takes columns half*128 .. +128 of each 256-column chunk (32 tokens when G = 4).
+        const int ew = warp - 2, quad = ew >> 2, grp = quad >> 1, hf = quad & 1, sp = warp & 3;
         const uint32_t lane_addr = (uint32_t)(sp * 32) << 16;
-        float* offs = sm.epi + ew * bt.rpad_max;       // this warp's copy of the row offsets
+        float* offs = sm.epi + ew * 256;          // this warp's negated row offsets: [chunk][128]
+        float2* xch = reinterpret_cast<float2*>(sm.epi + 16 * 256);   // [parity][grp][sp][32]
         const float c = bt.sl2e;
-        int64_t j = 0;                           // this group's chunks so far
+        const uint64_t cc = pack2(c, c);
+        int64_t j = 0, gt = 0;                   // chunks and tiles of this group so far
         int prev = -1;
         bool ok = true;
         for (int64_t u = ub; u < ue && ok; ++u) {
@@ -547,73 +611,31 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const int key = un.i * 65536 + un.s;
             if (key != prev) {
                 __syncwarp();
-                for (int r = lane; r < sd.R_pad; r += 32)   // stored negated: exp2(c z - offset) = exp2(fma(z, c, -offset))
-                    offs[r] = r < sd.R ? -sd.offs[(int64_t)un.s * sd.R + r] : -INFINITY;
+                for (int k = lane; k < nch * 128; k += 32) {
+                    const int r = (k >> 7) * 256 + hf * 128 + (k & 127);
+                    offs[k] = r < sd.R ? -sd.offs[(int64_t)un.s * sd.R + r] : -INFINITY;
+                }
                 __syncwarp();
                 prev = key;
             }
             const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
             const bool valid = pos >= 0 && pos < sd.T;
-            uint64_t nacc2 = 0ull, bsum2 = 0ull;   // pairs of token partial sums
+            const bool all_valid = __all_sync(0xffffffffu, valid);
+            uint64_t nacc2[2] = {0ull, 0ull}, bsum2[2] = {0ull, 0ull};   // pairs of token partial sums
             for (int ci = 0; ci < nch && ok; ++ci) {
                 if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
                 ++j;
                 tc_fence_after();
-                const int ncol = min(256, sd.R_pad - 256 * ci);
-                const float* ofc = offs + 256 * ci;
-                const bool all_valid = __all_sync(0xffffffffu, valid);
-                const uint64_t cc = pack2(c, c);
+                const int ncol = min(128, min(256, sd.R_pad - 256 * ci) - hf * 128);   // this half's columns
+                const uint32_t ta = tmem + lane_addr + grp * 256 + hf * 128;
+                const float* ofc = offs + ci * 128;
+                // 32-column steps; sixteen epilogue warps hide the TMEM load latency
 #pragma unroll 1
-                for (int col = 0; col < ncol; col += 64) {
-                    float v0[32], v1[32];
-                    const uint32_t ta = tmem + lane_addr + grp * 256 + col;
-                    tmem_ld32(ta, v0);
-                    tmem_ld32(ta + 32, v1);
+                for (int col = 0; col < ncol; col += 32) {
+                    float v[32];
+                    tmem_ld32(ta + col, v);
                     tmem_wait_ld();
-                    const float4* of4 = reinterpret_cast<const float4*>(ofc + col);
-                    float e[64];
-#pragma unroll
-                    for (int q = 0; q < 16; ++q) {
-                        const float4 o = of4[q];
-                        const int qb = 4 * (q & 7);
-                        const float z0 = q < 8 ? v0[qb] : v1[qb], z1 = q < 8 ? v0[qb + 1] : v1[qb + 1];
-                        const float z2 = q < 8 ? v0[qb + 2] : v1[qb + 2], z3 = q < 8 ? v0[qb + 3] : v1[qb + 3];
-                        float a0, a1, a2, a3;
-                        unpack2(ffma2(pack2(z0, z1), cc, pack2(o.x, o.y)), a0, a1);
-                        unpack2(ffma2(pack2(z2, z3), cc, pack2(o.z, o.w)), a2, a3);
-                        e[4 * q] = ex2(a0);
-                        e[4 * q + 1] = ex2(a1);
-                        e[4 * q + 2] = ex2(a2);
-                        e[4 * q + 3] = ex2(a3);
-                    }
-                    // b for the 64 / G tokens of these columns (a / G summed over the group's heads)
-                    constexpr int NT = 64 / G;
-                    float b[NT];
-#pragma unroll
-                    for (int k = 0; k < NT; ++k) {
-                        if (G == 1) b[k] = e[k];
-                        if (G == 2) b[k] = e[2 * k] + e[2 * k + 1];
-                        if (G == 4) {
-                            float x0, x1;
-                            unpack2(fadd2(pack2(e[4 * k], e[4 * k + 1]), pack2(e[4 * k + 2], e[4 * k + 3])), x0, x1);
-                            b[k] = x0 + x1;
-                        }
-                    }
-                    if (!all_valid) {
-#pragma unroll
-                        for (int k = 0; k < NT; ++k) b[k] = valid ? b[k] : 0.f;
-                    }
-#pragma unroll
-                    for (int k = 0; k < NT; k += 2) {
-                        const float p0 = lane_pool<PH>(b[k]), p1 = lane_pool<PH>(b[k + 1]);
-                        bsum2 = fadd2(bsum2, pack2(b[k], b[k + 1]));
-                        if (P2) {
-                            const uint64_t pp = pack2(p0, p1);
-                            nacc2 = ffma2(pp, pp, nacc2);
-                        } else {
-                            nacc2 = fadd2(nacc2, pack2(pow_p<false>(p0, bt.p), pow_p<false>(p1, bt.p)));
-                        }
-                    }
+                    accum_block<G, PH, P2>(v, ofc + col, cc, valid, all_valid, bt.p, nacc2, bsum2);
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -621,18 +643,33 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             }
             if (!ok) break;
             float nacc, bsum, t0_, t1_;
-            unpack2(nacc2, t0_, t1_);
+            unpack2(fadd2(nacc2[0], nacc2[1]), t0_, t1_);
             nacc = t0_ + t1_;
-            unpack2(bsum2, t0_, t1_);
+            unpack2(fadd2(bsum2[0], bsum2[1]), t0_, t1_);
             bsum = t0_ + t1_;
-            const float inv_m = 1.f / (float)sd.m;
-            const float pb = lane_pool<PH>(bsum * inv_m);
-            if (valid && lane >= kMargin && lane < kMargin + kOutW) {
-                const int64_t nS = (int64_t)bt.nL * bt.Hkv;
-                sd.part[(0 * nS + un.s) * sd.T + pos] = bsum * inv_m / (float)bt.Hkv;
-                sd.part[(1 * nS + un.s) * sd.T + pos] = nacc * inv_m;
-                sd.part[(2 * nS + un.s) * sd.T + pos] = pow_p<P2>(pb, bt.p);
+            // the two column halves of the group add up their sums; half 0 writes the results
+            const int tp = (int)(gt & 1);
+            float2* xs = xch + ((tp * 2 + grp) * 4 + sp) * 32;
+            uint64_t* xb = &ctl->xb[tp][grp][sp];
+            if (hf == 1) {
+                xs[lane] = make_float2(nacc, bsum);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(xb);
+            } else {
+                if (!(ok = wait_bar(xb, (uint32_t)((gt >> 1) & 1), ctl, bt.err, 14))) break;
+                const float2 o = xs[lane];
+                nacc += o.x;
+                bsum += o.y;
+                const float inv_m = 1.f / (float)sd.m;
+                const float pb = lane_pool<PH>(bsum * inv_m);
+                if (valid && lane >= kMargin && lane < kMargin + kOutW) {
+                    const int64_t nS = (int64_t)bt.nL * bt.Hkv;
+                    sd.part[(0 * nS + un.s) * sd.T + pos] = bsum * inv_m / (float)bt.Hkv;
+                    sd.part[(1 * nS + un.s) * sd.T + pos] = nacc * inv_m;
+                    sd.part[(2 * nS + un.s) * sd.T + pos] = pow_p<P2>(pb, bt.p);
+                }
             }
+            ++gt;
         }
     }
     tc_fence_before();
@@ -671,7 +708,7 @@ bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4], const
 }
 
 size_t smem_bytes(int rpad_max, int stages) {
-    return 1024 + (size_t)2 * rpad_max * 128 + (size_t)stages * kTileBytes + 256 + (size_t)8 * rpad_max * 4;
+    return 1024 + (size_t)2 * rpad_max * 128 + (size_t)stages * kTileBytes + 512 + 16 * 256 * 4 + 2 * 2 * 4 * 32 * 8;
 }
 
 template <int G, int PH, bool P2>
@@ -739,13 +776,13 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             d.R = s.m * G;
             d.R_pad = (d.R + 127) / 128 * 128;
             rpad_max = rpad_max > d.R_pad ? rpad_max : d.R_pad;
-            d.n_chunk1 = (int32_t)(2 * ((s.T + kChunk1 - 1) / kChunk1));   // one partial per (chunk, group)
+            d.n_chunk1 = (int32_t)(4 * ((s.T + kChunk1 - 1) / kChunk1));   // one partial per (chunk, group, half)
             d.n_tile2 = (int32_t)((s.T + kOut2 - 1) / kOut2);
             d.stats = b.stats + s.stats_off;
             d.offs = b.offs + s.offs_off;
             d.part = b.part + s.part_off;
             d.unit1_begin = u1;
-            u1 += (int64_t)nS * (d.n_chunk1 / 2);
+            u1 += (int64_t)nS * (d.n_chunk1 / 4);
             d.unit2_begin = u2;
             u2 += (int64_t)nS * d.n_tile2;
             // Q arrives in boxes of at most 256 tokens that tile the padded rows exactly

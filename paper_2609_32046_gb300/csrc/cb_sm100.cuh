@@ -82,6 +82,14 @@ __device__ __forceinline__ void tma_load_4d(void* smem, const CUtensorMap* m, ui
         : "memory");
 }
 
+// Prefetch a tensor tile into L2 (no shared memory, no completion tracking).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* m, int32_t x, int32_t y, int32_t z, int32_t w) {
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(x), "r"(y), "r"(z), "r"(w)
+                 : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // tcgen05: tensor memory
 // ---------------------------------------------------------------------------
@@ -212,6 +220,16 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     float r;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
     return r;
+}
+
+// Max of 32 register values by a tree of 3-input max.
+__device__ __forceinline__ float max_tree1(const float (&x)[32]) {
+    float u[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) u[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
+    u[10] = fmaxf(x[30], x[31]);
+    const float w0 = fmax3(u[0], u[1], u[2]), w1 = fmax3(u[3], u[4], u[5]), w2 = fmax3(u[6], u[7], u[8]);
+    return fmax3(w0, w1, fmax3(w2, u[9], u[10]));
 }
 
 // Max of two 32-value register arrays by a tree of 3-input max (depth 4).
