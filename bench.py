@@ -67,34 +67,92 @@ def workload_bytes_flops(spec, keep):
     return tot_b, score_b, compact_b, tot_f
 
 
-class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled in the background."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
-         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-         "clocks_event_reasons.sw_power_cap")
+_REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+            0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, index: int):
-        self.index = index
-        self.samples = []
-        self.proc = None
+
+class ClockSampler:
+    """SM clock, power and clock-event (throttle) reasons sampled every 2 ms through NVML
+    (read-only queries), falling back to `nvidia-smi -lms 50`."""
+
+    def __init__(self, cuda_index: int):
+        self.cuda_index = cuda_index
+        self.samples = []          # (time, sm_mhz, reasons_bitmask or names, power_w)
+        self.sm_max = None
+        self._stop = threading.Event()
         self.thread = None
+        self.proc = None
+        self.source = None
+
+    def _nvml_handle(self):
+        import ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        try:
+            import torch
+            pr = torch.cuda.get_device_properties(self.cuda_index)
+            bus = b"%08x:%02x:%02x.0" % (pr.pci_domain_id, pr.pci_bus_id, pr.pci_device_id)
+            if lib.nvmlDeviceGetHandleByPciBusId_v2(bus, ctypes.byref(h)) != 0:
+                raise OSError("no handle for %r" % bus)
+        except Exception:
+            if lib.nvmlDeviceGetHandleByIndex_v2(self.cuda_index, ctypes.byref(h)) != 0:
+                raise OSError("no NVML handle")
+        return lib, h
+
+    def _nvml_loop(self, lib, h):
+        import ctypes
+        mhz, mw, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        get_reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        while not self._stop.is_set():
+            t = time.time()
+            lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz))      # NVML_CLOCK_SM
+            get_reasons(h, ctypes.byref(rs))
+            lib.nvmlDeviceGetPowerUsage(h, ctypes.byref(mw))
+            self.samples.append((t, float(mhz.value), int(rs.value), mw.value / 1000.0))
+            time.sleep(0.002)
 
     def start(self):
         try:
-            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+            import ctypes
+            lib, h = self._nvml_handle()
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.sm_max = float(mx.value)
+            self.source = "nvml, 2 ms"
+            self.thread = threading.Thread(target=self._nvml_loop, args=(lib, h), daemon=True)
+            self.thread.start()
+            return
+        except Exception:
+            pass
+        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.cuda_index), "--query-gpu=" + q,
                                           "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
-            self.proc = None
             return
-        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.source = "nvidia-smi, 50 ms"
+
+        def read():
+            names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+            for line in self.proc.stdout:
+                parts = [x.strip() for x in line.split(",")]
+                try:
+                    self.sm_max = float(parts[1])
+                    act = [names[k] for k in range(4) if parts[3 + k].lower() == "active"]
+                    self.samples.append((time.time(), float(parts[0]), act, float(parts[2])))
+                except (ValueError, IndexError):
+                    pass
+        self.thread = threading.Thread(target=read, daemon=True)
         self.thread.start()
 
-    def _read(self):
-        for line in self.proc.stdout:
-            self.samples.append((time.time(), line.strip()))
-
     def stop(self):
+        self._stop.set()
         if self.proc:
             self.proc.terminate()
             try:
@@ -105,33 +163,41 @@ class ClockSampler:
             self.thread.join(timeout=2)
 
     def summary(self, t0, t1):
-        rows = []
-        for ts, line in self.samples:
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
-                continue
-            rows.append((ts, parts))
-        window = [r for r in rows if t0 <= r[0] <= t1]
+        window = [x for x in self.samples if t0 <= x[0] <= t1]
         note = "in timed region"
         if not window:
-            # the timed region was shorter than the sampling period: take the samples nearest it
-            window = sorted(rows, key=lambda r: min(abs(r[0] - t0), abs(r[0] - t1)))[:3]
-            note = "nearest samples (timed region shorter than the 50 ms sampling period)"
+            window = sorted(self.samples, key=lambda x: min(abs(x[0] - t0), abs(x[0] - t1)))[:3]
+            note = "nearest samples to the timed region"
         if not window:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+            return {"sm_mhz": None, "sm_max_mhz": self.sm_max, "reasons": ["unsampled"], "samples": 0}
+        reasons = set()
+        for _, _, r, _ in window:
+            if isinstance(r, int):
+                reasons |= {name for bit, name in _REASONS.items() if r & bit}
+            else:
+                reasons |= set(r)
+        return {"sm_mhz": statistics.median([x[1] for x in window]), "sm_max_mhz": self.sm_max,
+                "reasons": sorted(reasons), "samples": len(window), "note": note, "source": self.source,
+                "power_w_max": max(x[3] for x in window)}
 
-        def num(x):
-            try:
-                return float(x)
-            except ValueError:
-                return None
-        sm = [num(p[1]) for _, p in window if num(p[1]) is not None]
-        smax = [num(p[2]) for _, p in window if num(p[2]) is not None]
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[k] for _, p in window for k in range(4) if p[5 + k].lower() == "active"})
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "reasons": reasons, "samples": len(window), "note": note,
-                "power_w_max": max((num(p[3]) or 0.0) for _, p in window)}
+
+def traffic_for(kernel: str, workload: str):
+    """DRAM bytes (read + write) per launch of `kernel` on `workload` from the committed ncu
+    summary, or None when that summary was taken on a different build of the kernel source."""
+    import hashlib
+    import re
+    path = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
+    src = os.path.join(ROOT, "paper_2609_32046_gb300", "csrc", "cb_score_tc.cu")
+    try:
+        text = open(path).read()
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+        m_tr = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
+        if m_sha and m_tr and m_sha.group(1) == sha:
+            return int(m_tr.group(1))
+    except OSError:
+        pass
+    return None
 
 
 def dist_init():
@@ -257,12 +323,13 @@ def run_ours(args):
                      spec.m, max(spec.T), len(senders))
     f = cb.Filter(c, senders, queries, keep, device=dev)
     stream = torch.cuda.current_stream(dev)
-    n_launch_per_step = 6 * math.ceil(len(senders) / 64)
 
     for _ in range(args.warmup):
         f.run(stream)
     c.sync_status(stream)
 
+    c.enable_stage_timing(True)
+    c.stage_times()                                  # reset the sums
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(4 * args.steps)]
     sampler = ClockSampler(local)
     sampler.start()
@@ -287,6 +354,9 @@ def run_ours(args):
     barrier(ws)
     sampler.stop()
     c.sync_status(stream)
+    stage_ms, stage_calls = c.stage_times()
+    c.enable_stage_timing(False)
+    stage_avg = {k: v / max(1, stage_calls) for k, v in stage_ms.items()}
     ms = start.elapsed_time(end)
     ms_max = max_over_ranks(ws, ms)
     per = {"score": [], "select": [], "compact": []}
@@ -297,9 +367,15 @@ def run_ours(args):
     avg = {k: sum(v) / len(v) for k, v in per.items()}
 
     tokens_per_rank = sum(f.Ts)
+    n_send = len(senders)
+    score_batches = math.ceil(n_send / 64)
+    tc_batches = sum(math.ceil(min(64, n_send - 64 * b) / 32) for b in range(score_batches))
+    launches_per_step = (3 * tc_batches + score_batches) + 2 * score_batches   # score kernels, select, compact
     value = tokens_per_rank * ws * args.steps / (ms_max / 1e3)
     hbm_peak, tc_peak, tc_sus, src = peaks()
     tot_b, score_b, compact_b, flops = workload_bytes_flops(spec, keep)
+    pass_flops = flops / 2                                   # one QK^T pass
+    part_bytes = sum(3 * spec.shape.n_layers * spec.shape.n_kv_heads * T * 4 for T in f.Ts)
     step_s = ms / args.steps / 1e3
 
     # e2e: the same step through the C-ABI with the inputs in pinned host memory
@@ -359,16 +435,31 @@ def run_ours(args):
         "algorithmic_bytes_per_step": tot_b,
         "step_ms": {k: v for k, v in avg.items()},
         "roofline": {
-            "bound": "tensor", "kernel": "score (stats + accumulate passes)",
-            "achieved": flops / (avg["score"] / 1e3) / 1e12, "peak": tc_peak, "unit": "TFLOP/s",
-            "frac": flops / (avg["score"] / 1e3) / 1e12 / tc_peak, "traffic": None,
-            "peak_source": "%s bf16 burst" % src,
+            "bound": "tensor", "kernel": "k_accum_tc (normalised accumulation: second QK^T pass + epilogue)",
+            "achieved": pass_flops / (stage_avg["normalised_accumulation"] / 1e3) / 1e12, "peak": tc_peak,
+            "unit": "TFLOP/s", "frac": pass_flops / (stage_avg["normalised_accumulation"] / 1e3) / 1e12 / tc_peak,
+            "traffic": traffic_for("k_accum_tc", args.workload),
+            "peak_source": "%s bf16 burst (cuBLAS)" % src,
+            "algorithmic_flops_per_launch": pass_flops,
         },
-        "roofline_compact": {
-            "bound": "hbm", "achieved": compact_b / (avg["compact"] / 1e3) / 1e9, "peak": hbm_peak, "unit": "GB/s",
-            "frac": compact_b / (avg["compact"] / 1e3) / 1e9 / hbm_peak, "peak_source": "%s copy" % src,
+        "kernels": {
+            "row_statistics": {"ms": stage_avg["row_statistics"], "bound": "tensor",
+                               "tflops": pass_flops / (stage_avg["row_statistics"] / 1e3) / 1e12},
+            "normalised_accumulation": {"ms": stage_avg["normalised_accumulation"], "bound": "tensor",
+                                        "tflops": pass_flops / (stage_avg["normalised_accumulation"] / 1e3) / 1e12},
+            "statistics_combine": {"ms": stage_avg["statistics_combine"]},
+            "finalize": {"ms": stage_avg["finalize"], "bound": "hbm",
+                         "gbs": part_bytes / (stage_avg["finalize"] / 1e3) / 1e9},
+            "select": {"ms": avg["select"]},
+            "compact": {"ms": avg["compact"], "bound": "hbm", "gbs": compact_b / (avg["compact"] / 1e3) / 1e9,
+                        "frac": compact_b / (avg["compact"] / 1e3) / 1e9 / hbm_peak},
         },
-        "gpu_launches": n_launch_per_step * args.steps,
+        "roofline_step": {
+            "t_hbm_us": tot_b / (hbm_peak * 1e9) * 1e6, "t_tensor_us": flops / (tc_peak * 1e12) * 1e6,
+            "frac": max(tot_b / (hbm_peak * 1e9), flops / (tc_peak * 1e12)) / step_s,
+            "note": "max(HBM time of the algorithmic bytes, tensor time of both QK^T passes) / step time",
+        },
+        "gpu_launches": launches_per_step * args.steps,
         "clocks": sampler.summary(t_wall0, t_wall1),
     }
     if e2e:

@@ -164,6 +164,18 @@ cb_status cb_compact(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t
  * (CB_EDEVICE) or a failed launch (CB_ECUDA).  Blocks the host. */
 cb_status cb_sync_status(cb_ctx *ctx, void *stream);
 
+/*
+ * Per-kernel timing of cb_score (tracing).  While enabled, every cb_score records CUDA events on
+ * its stream between its internal kernels (no synchronisation, a few microseconds of overhead).
+ * cb_stage_times waits for the last recorded event and writes, into ms[0..3], the summed
+ * milliseconds since the previous read of the four score kernels: row statistics (first logit
+ * pass), statistics combine, normalised accumulation (second logit pass), finalize; *calls
+ * receives the number of cb_score calls covered.  The sums are then reset.  Errors: CB_EINVAL
+ * (timing not enabled, NULL arguments), CB_ECUDA.
+ */
+cb_status cb_enable_stage_timing(cb_ctx *ctx, int32_t enable);
+cb_status cb_stage_times(cb_ctx *ctx, float *ms, int32_t *calls);
+
 /* Free the context's scratch (after synchronising its device).  NULL is ignored. */
 void cb_destroy(cb_ctx *ctx);
 

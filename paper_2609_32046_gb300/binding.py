@@ -20,7 +20,8 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
-            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_select_noalloc"]
+            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_select_noalloc",
+            "cb_enable_stage_timing", "cb_stage_times"]
 
 
 class CBError(RuntimeError):
@@ -86,6 +87,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_scratch_bytes.restype = ctypes.c_int64
     lib.cb_select_noalloc.argtypes = [ctypes.c_int32, P, P, P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
     lib.cb_select_noalloc.restype = ctypes.c_int
+    lib.cb_enable_stage_timing.argtypes = [P, ctypes.c_int32]
+    lib.cb_enable_stage_timing.restype = ctypes.c_int
+    lib.cb_stage_times.argtypes = [P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int32)]
+    lib.cb_stage_times.restype = ctypes.c_int
     if path is None:
         _LIB = lib
     return lib
@@ -208,6 +213,18 @@ class CacheBack:
         self._check(self.lib.cb_compact(self.h, n, kv, ip, Ba, k_out.data_ptr(), v_out.data_ptr(),
                                         k_out.shape[2], Oa, k_out.stride(0), k_out.stride(1),
                                         _stream_handle(stream)))
+
+    STAGES = ("row_statistics", "statistics_combine", "normalised_accumulation", "finalize")
+
+    def enable_stage_timing(self, enable: bool = True):
+        self._check(self.lib.cb_enable_stage_timing(self.h, 1 if enable else 0))
+
+    def stage_times(self):
+        """(dict stage -> summed ms, number of cb_score calls) since the previous read."""
+        ms = (ctypes.c_float * 4)()
+        calls = ctypes.c_int32()
+        self._check(self.lib.cb_stage_times(self.h, ms, ctypes.byref(calls)))
+        return dict(zip(self.STAGES, list(ms))), int(calls.value)
 
     def sync_status(self, stream=None):
         self._check(self.lib.cb_sync_status(self.h, _stream_handle(stream)))

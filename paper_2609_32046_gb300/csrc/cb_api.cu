@@ -16,6 +16,33 @@
 #include "cacheback.h"
 #include "cb_internal.cuh"
 
+namespace cbk {
+// Events recorded around each score kernel while stage timing is enabled.  Each mark closes
+// the interval that started at the previous mark; intervals are summed per stage on read.
+struct StageTimer {
+    std::vector<cudaEvent_t> pool;                 // created once, reused after each read
+    std::vector<std::pair<int, cudaEvent_t>> marks;
+    size_t used = 0;
+    int calls = 0;
+    ~StageTimer() {
+        for (cudaEvent_t e : pool) cudaEventDestroy(e);
+    }
+};
+
+void stage_mark(StageTimer* t, int stage, cudaStream_t st) {
+    if (!t) return;
+    if (t->used == t->pool.size()) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) { cudaGetLastError(); return; }
+        t->pool.push_back(e);
+    }
+    cudaEvent_t e = t->pool[t->used++];
+    if (cudaEventRecord(e, st) != cudaSuccess) { cudaGetLastError(); return; }
+    t->marks.emplace_back(stage, e);
+    if (stage == kStageStart) ++t->calls;
+}
+}  // namespace cbk
+
 struct cb_ctx {
     cb_config cfg;
     int device = 0;
@@ -31,6 +58,7 @@ struct cb_ctx {
     uint32_t* err = nullptr;
     int64_t keys_per_sender = 0;
     int64_t scratch_bytes = 0;
+    cbk::StageTimer* timer = nullptr;
     std::string last_error;
 };
 
@@ -210,6 +238,7 @@ void cb_destroy(cb_ctx* ctx) {
         cudaFree(ctx->part);
         cudaFree(ctx->span_keys);
         cudaFree(ctx->err);
+        delete ctx->timer;
     }
     delete ctx;
 }
@@ -255,6 +284,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->alpha = c.alpha;
         bt->pool_half = c.pool_width / 2;
         bt->use_tc = ctx->use_tc ? 1 : 0;
+        bt->timer = ctx->timer;
         bt->err = ctx->err;
         bt->stats = ctx->stats;
         bt->offs = ctx->offs;
@@ -395,6 +425,46 @@ cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t
         cudaError_t e = cbk::launch_compact(bt, strm, ctx->num_sms);
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "compact launch failed: %s", cudaGetErrorString(e));
     }
+    return CB_OK;
+}
+
+cb_status cb_enable_stage_timing(cb_ctx* ctx, int32_t enable) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    DeviceGuard dg(ctx->device);
+    if (enable && !ctx->timer) ctx->timer = new cbk::StageTimer();
+    if (!enable && ctx->timer) {
+        cudaDeviceSynchronize();
+        delete ctx->timer;
+        ctx->timer = nullptr;
+    }
+    return CB_OK;
+}
+
+cb_status cb_stage_times(cb_ctx* ctx, float* ms, int32_t* calls) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    if (!ms || !calls) return fail(ctx, CB_EINVAL, "ms or calls is NULL");
+    for (int k = 0; k < 4; ++k) ms[k] = 0.f;
+    *calls = 0;
+    cbk::StageTimer* t = ctx->timer;
+    if (!t) return fail(ctx, CB_EINVAL, "stage timing is not enabled");
+    DeviceGuard dg(ctx->device);
+    if (!t->marks.empty()) {
+        cudaError_t e = cudaEventSynchronize(t->marks.back().second);
+        if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "event wait failed: %s", cudaGetErrorString(e));
+        for (size_t i = 1; i < t->marks.size(); ++i) {
+            const int stage = t->marks[i].first;
+            if (stage == cbk::kStageStart) continue;
+            float x = 0.f;
+            if (cudaEventElapsedTime(&x, t->marks[i - 1].second, t->marks[i].second) == cudaSuccess)
+                ms[stage - 1] += x;
+            else
+                cudaGetLastError();
+        }
+    }
+    *calls = t->calls;
+    t->marks.clear();
+    t->used = 0;
+    t->calls = 0;
     return CB_OK;
 }
 

@@ -28,6 +28,12 @@ constexpr uint32_t kErrCompactIndex = 1u;
 constexpr uint32_t kErrSelectBudget = 2u;
 constexpr uint32_t kErrTimeout = 4u;       // a bounded mbarrier wait gave up
 
+// Optional per-kernel timing of the score step (owned by the context; see cb_stage_times).
+struct StageTimer;
+enum ScoreStage { kStageStart = 0, kStageStats = 1, kStageCombine = 2, kStageAccum = 3, kStageFinalize = 4 };
+// Records an event on `st` marking the end of `stage` (no-op when timer is null).
+void stage_mark(StageTimer* timer, int stage, cudaStream_t st);
+
 struct ScoreSender {
     const uint16_t* k;        // K[l][g][t][:] at k + l*ks_l + g*ks_h + t*ks_p
     const uint16_t* q;        // Q[l][r][h][:] at q + l*qs_l + r*qs_t + h*qs_h
@@ -54,6 +60,7 @@ struct ScoreBatch {
     int32_t pool_half;        // pool_width / 2
     int32_t use_tc;           // 1: tcgen05 passes, 0: mma.sync passes
     uint32_t* err;            // device error word
+    StageTimer* timer;        // host-side; null unless stage timing is enabled
     float2* stats;            // pass-1 partial (max, sum) in log2 domain
     float* offs;              // per-row log2 offsets (max + log2(sum) + log2(G))
     float* part;              // per-group U_s, N_s, D_s partials

@@ -477,10 +477,15 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(k_accum<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
     if (e != cudaSuccess) return e;
+    stage_mark(b.timer, kStageStart, st);
     k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
+    stage_mark(b.timer, kStageStats, st);
     k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
+    stage_mark(b.timer, kStageCombine, st);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
+    stage_mark(b.timer, kStageAccum, st);
     k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(b);
+    stage_mark(b.timer, kStageFinalize, st);
     return cudaGetLastError();
 }
 
@@ -516,6 +521,7 @@ cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
             int64_t nblkf = 0;
             for (int i = 0; i < w->n; ++i) nblkf += finalize_blocks(w->s[i].T);
             k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(*w);
+            stage_mark(w->timer, kStageFinalize, st);
             e = cudaGetLastError();
         }
         delete w;

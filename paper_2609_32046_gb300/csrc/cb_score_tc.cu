@@ -820,7 +820,9 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         e = cudaFuncSetAttribute(k_stats_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e == cudaSuccess) {
             const int g1 = (int)(tb->units1 < num_sms ? tb->units1 : num_sms);
+            stage_mark(b.timer, kStageStart, st);
             k_stats_tc<<<g1, kThreadsTc, smem, st>>>(*tb);
+            stage_mark(b.timer, kStageStats, st);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) {
@@ -832,6 +834,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
                 sub->s[j].n_chunk1 = tb->s[j].n_chunk1;
             }
             e = combine(*sub, st);
+            stage_mark(b.timer, kStageCombine, st);
             delete sub;
         }
         if (e == cudaSuccess) {
@@ -839,6 +842,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             if (G == 4) e = launch_accum_g<4>(*tb, smem, g2, st);
             else if (G == 2) e = launch_accum_g<2>(*tb, smem, g2, st);
             else e = launch_accum_g<1>(*tb, smem, g2, st);
+            stage_mark(b.timer, kStageAccum, st);
         }
     }
     free_all();
