@@ -54,6 +54,7 @@ struct cb_ctx {
     float2* stats = nullptr;
     float* offs = nullptr;
     float* part = nullptr;
+    float* fin = nullptr;
     float* span_keys = nullptr;
     uint32_t* err = nullptr;
     int64_t keys_per_sender = 0;
@@ -214,6 +215,7 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     e = alloc(&ctx->stats, (size_t)(S * nS * ctx->n_chunk1_max * rows), &total);
     if (e == cudaSuccess) e = alloc(&ctx->offs, (size_t)(S * nS * rows), &total);
     if (e == cudaSuccess) e = alloc(&ctx->part, (size_t)(S * 3 * nS * c.max_positions), &total);
+    if (e == cudaSuccess) e = alloc(&ctx->fin, (size_t)(S * cbk::kFinSlices * 3 * c.max_positions), &total);
     if (e == cudaSuccess) e = alloc(&ctx->span_keys, (size_t)(S * ctx->keys_per_sender), &total);
     if (e == cudaSuccess) e = alloc(&ctx->err, 1, &total);
     if (e == cudaSuccess) e = cudaMemset(ctx->err, 0, sizeof(uint32_t));
@@ -236,6 +238,7 @@ void cb_destroy(cb_ctx* ctx) {
         cudaFree(ctx->stats);
         cudaFree(ctx->offs);
         cudaFree(ctx->part);
+        cudaFree(ctx->fin);
         cudaFree(ctx->span_keys);
         cudaFree(ctx->err);
         delete ctx->timer;
@@ -289,7 +292,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->stats = ctx->stats;
         bt->offs = ctx->offs;
         bt->part = ctx->part;
-        int64_t so = 0, oo = 0, po = 0, b1 = 0, b2 = 0;
+        bt->fin = ctx->fin;
+        int64_t so = 0, oo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
             const cb_query& q = queries[b0 + k];
@@ -306,6 +310,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.stats_off = so; so += (int64_t)nS * cbk::stats_slots(s.T) * q.m * ctx->G;
             d.offs_off = oo; oo += (int64_t)nS * q.m * ctx->G;
             d.part_off = po; po += (int64_t)3 * nS * s.T;
+            d.fin_off = fo; fo += (int64_t)cbk::kFinSlices * 3 * s.T;
             d.blk1_begin = b1; b1 += (int64_t)nS * d.n_chunk1;
             d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
             d.blkf_begin = 0;  // set by the score launcher

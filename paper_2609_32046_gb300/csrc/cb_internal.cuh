@@ -9,7 +9,7 @@ namespace cbk {
 
 constexpr int kMaxBatch = 64;        // senders per launch (larger calls are split)
 constexpr int kStatsChunk = 256;     // positions per pass-1 block (mma.sync path)
-constexpr int kStatsChunkTc = 512;   // positions per pass-1 chunk (tcgen05 path, four partials each)
+constexpr int kStatsChunkTc = 1024;  // positions per pass-1 chunk (tcgen05 path, four partials each)
 
 // Pass-1 partial slots a sender of T positions may need on either path.
 inline int64_t stats_slots(int64_t T) {
@@ -21,6 +21,7 @@ constexpr int kAccumChunk = 128;     // output positions per pass-2 block
 constexpr int kHalo = 8;             // extra positions each side of a pass-2 block (>= pool_width/2)
 constexpr int kMaxPoolWidth = 15;
 constexpr int kMaxSpanWidth = 256;
+constexpr int kFinSlices = 16;        // finalize: groups summed in 16 fixed slices
 constexpr int kMaxQueryTokens = 1024;
 
 // Device error word bits (set by kernels' own bounds checks).
@@ -47,6 +48,7 @@ struct ScoreSender {
     int64_t stats_off;        // float2 offset of this sender's pass-1 partials
     int64_t offs_off;         // float offset of this sender's per-row softmax offsets
     int64_t part_off;         // float offset of this sender's [3][nS][T] partials
+    int64_t fin_off;          // float offset of this sender's [kFinSlices][3][T] slice sums
     int64_t blk1_begin;       // first pass-1 block of this sender
     int64_t blk2_begin;       // first pass-2 block of this sender
     int64_t blkf_begin;       // first finalize block of this sender
@@ -64,6 +66,7 @@ struct ScoreBatch {
     float2* stats;            // pass-1 partial (max, sum) in log2 domain
     float* offs;              // per-row log2 offsets (max + log2(sum) + log2(G))
     float* part;              // per-group U_s, N_s, D_s partials
+    float* fin;               // finalize slice sums [sender][kFinSlices][3][T]
     ScoreSender s[kMaxBatch];
 };
 

@@ -252,8 +252,10 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
     for (int row = threadIdx.x; row < R; row += kThreads) {
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
         float M = -INFINITY;
+#pragma unroll 8
         for (int c = 0; c < sd.n_chunk1; ++c) M = fmaxf(M, st[(int64_t)c * R].x);
         float L = 0.f;
+#pragma unroll 8
         for (int c = 0; c < sd.n_chunk1; ++c) {
             const float2 v = st[(int64_t)c * R];
             if (v.x != -INFINITY) L += v.y * ex2(v.x - M);
@@ -385,57 +387,58 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // finalize: fixed-order sums over the groups, Pool(U), C, S
 // ---------------------------------------------------------------------------
-constexpr int kFinSlices = 12;                          // groups s split over 12 threads per position
-constexpr int kFinPos = 80;                             // positions per block incl. 8-position halos
-constexpr int kFinOut2 = kFinPos - 2 * kHalo;           // 64 outputs per block
-
-__global__ void __launch_bounds__(kFinPos * kFinSlices) k_finalize(const __grid_constant__ ScoreBatch bt) {
-    __shared__ float red[3][kFinSlices][kFinPos];
-    __shared__ float us[kFinPos];
+// Stage 1: slice k of the groups (s = k, k + 16, ...) summed in increasing order per position.
+__global__ void __launch_bounds__(256) k_fin_sum(const __grid_constant__ ScoreBatch bt) {
     const int nS = bt.n_layers * bt.n_kv_heads;
+    const ScoreSender& sd = bt.s[blockIdx.z];
+    const int sl = blockIdx.y;
+    const int64_t T = sd.T;
+    const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
+    if (t >= T) return;
+    const float* part = bt.part + sd.part_off + t;
+    float U = 0.f, Nv = 0.f, Dv = 0.f;
+#pragma unroll 6
+    for (int s = sl; s < nS; s += kFinSlices) {
+        U += __ldcs(part + (int64_t)s * T);
+        Nv += __ldcs(part + ((int64_t)nS + s) * T);
+        Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
+    }
+    float* fin = bt.fin + sd.fin_off + (int64_t)sl * 3 * T + t;
+    fin[0] = U;
+    fin[T] = Nv;
+    fin[2 * T] = Dv;
+}
+
+// Stage 2: the 16 slice sums in fixed order, Pool(U) through shared memory, C and S.
+constexpr int kFinBlock = 256;
+constexpr int kFinOut2 = kFinBlock - 2 * kHalo;        // outputs per block
+
+__global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ ScoreBatch bt) {
+    __shared__ float us[kFinBlock];
     const int64_t blk = blockIdx.x;
     const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blkf_begin; });
     const ScoreSender& sd = bt.s[i];
     const int64_t T = sd.T;
-    const int lp = threadIdx.x % kFinPos, sl = threadIdx.x / kFinPos;
+    const int lp = threadIdx.x;
     const int64_t t = (blk - sd.blkf_begin) * kFinOut2 - kHalo + lp;
     const bool inside = (t >= 0 && t < T);
-    const bool centre = lp >= kHalo && lp < kFinPos - kHalo;
-    const float* part = bt.part + sd.part_off;
+    const bool centre = lp >= kHalo && lp < kFinBlock - kHalo;
+    const float* fin = bt.fin + sd.fin_off + t;
     float U = 0.f, Nv = 0.f, Dv = 0.f;
     if (inside) {
-        // slice sl adds groups sl, sl + 12, ... in increasing order
-        const float* pu = part + t;
-#pragma unroll 8
-        for (int s = sl; s < nS; s += kFinSlices) U += __ldcs(pu + (int64_t)s * T);
+#pragma unroll
+        for (int k = 0; k < kFinSlices; ++k) U += fin[(int64_t)k * 3 * T];
         if (centre) {
-            const float* pn = part + (int64_t)nS * T + t;
-            const float* pd = part + (int64_t)2 * nS * T + t;
-#pragma unroll 8
-            for (int s = sl; s < nS; s += kFinSlices) {
-                Nv += __ldcs(pn + (int64_t)s * T);
-                Dv += __ldcs(pd + (int64_t)s * T);
+#pragma unroll
+            for (int k = 0; k < kFinSlices; ++k) {
+                Nv += fin[((int64_t)k * 3 + 1) * T];
+                Dv += fin[((int64_t)k * 3 + 2) * T];
             }
         }
     }
-    red[0][sl][lp] = U;
-    red[1][sl][lp] = Nv;
-    red[2][sl][lp] = Dv;
+    us[lp] = U;
     __syncthreads();
-    if (sl == 0) {
-        U = red[0][0][lp];
-        Nv = red[1][0][lp];
-        Dv = red[2][0][lp];
-#pragma unroll
-        for (int k = 1; k < kFinSlices; ++k) {   // fixed order: deterministic
-            U += red[0][k][lp];
-            Nv += red[1][k][lp];
-            Dv += red[2][k][lp];
-        }
-        us[lp] = U;
-    }
-    __syncthreads();
-    if (sl == 0 && centre && inside) {
+    if (centre && inside) {
         const int ph = bt.pool_half;
         float Q = us[lp - ph];
         for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[lp + u]);
@@ -443,6 +446,18 @@ __global__ void __launch_bounds__(kFinPos * kFinSlices) k_finalize(const __grid_
         const float S = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
         sd.scores[t] = S;
     }
+}
+
+cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
+    int64_t maxT = 0, nblk = 0;
+    for (int i = 0; i < b.n; ++i) {
+        maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
+        nblk += (b.s[i].T + kFinOut2 - 1) / kFinOut2;
+    }
+    dim3 g1((unsigned)((maxT + 255) / 256), kFinSlices, (unsigned)b.n);
+    k_fin_sum<<<g1, 256, 0, st>>>(b);
+    k_finalize<<<(unsigned)nblk, kFinBlock, 0, st>>>(b);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
@@ -453,6 +468,7 @@ cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
 }
 
 int64_t finalize_blocks(int64_t T) { return (T + kFinOut2 - 1) / kFinOut2; }
+
 
 template <int D, int G>
 size_t accum_smem(int max_rows) {
@@ -484,7 +500,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     stage_mark(b.timer, kStageCombine, st);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
     stage_mark(b.timer, kStageAccum, st);
-    k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(b);
+    launch_finalize(b, st);
     stage_mark(b.timer, kStageFinalize, st);
     return cudaGetLastError();
 }
@@ -518,9 +534,7 @@ cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
             return e;
         }
         if (e == cudaSuccess) {
-            int64_t nblkf = 0;
-            for (int i = 0; i < w->n; ++i) nblkf += finalize_blocks(w->s[i].T);
-            k_finalize<<<(unsigned)nblkf, kFinPos * kFinSlices, 0, st>>>(*w);
+            launch_finalize(*w, st);
             stage_mark(w->timer, kStageFinalize, st);
             e = cudaGetLastError();
         }
