@@ -62,6 +62,7 @@ struct TcSender {
     int32_t m, R, R_pad;
     int32_t n_chunk1, n_tile2;
     int32_t qbox_tok, n_qbox;
+    float inv_m, inv_mh;  // 1 / m and 1 / (m Hkv)
     int64_t unit1_begin, unit2_begin;
 };
 
@@ -140,6 +141,30 @@ __device__ __forceinline__ Unit decode2(const TcBatch& bt, int64_t u) {
     while (i + 1 < bt.n && bt.s[i + 1].unit2_begin <= u) ++i;
     const int64_t local = u - bt.s[i].unit2_begin;
     return Unit{i, (int)(local / bt.s[i].n_tile2), (int)(local % bt.s[i].n_tile2)};
+}
+
+// Pass-2 units in order without a division per unit: (sender, group, tile) advanced by one.
+__device__ __forceinline__ void next2(const TcBatch& bt, Unit& un) {
+    if (un.i >= bt.n) return;   // past the last unit
+    if (++un.c == bt.s[un.i].n_tile2) {
+        un.c = 0;
+        if (++un.s == bt.nL * bt.Hkv) {
+            un.s = 0;
+            ++un.i;
+        }
+    }
+}
+
+// Pass-1 units likewise (sender, group, chunk).
+__device__ __forceinline__ void next1(const TcBatch& bt, Unit& un) {
+    if (un.i >= bt.n) return;
+    if (++un.c == bt.s[un.i].n_chunk1 / 4) {
+        un.c = 0;
+        if (++un.s == bt.nL * bt.Hkv) {
+            un.s = 0;
+            ++un.i;
+        }
+    }
 }
 
 // Contiguous share of `total` units for this CTA.
@@ -293,8 +318,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
             int64_t kt = 0, qn = 0;
             int prev = -1;
             bool ok = true;
-            for (int64_t u = ub; u < ue && ok; ++u) {
-                const Unit un = decode1(bt, u);
+            Unit un = decode1(bt, ub);
+            for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
                 const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
                 const int key = un.i * 65536 + un.s;
@@ -323,8 +348,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
             int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
             int prev = -1;
             bool ok = true;
-            for (int64_t u = ub; u < ue && ok; ++u) {
-                const Unit un = decode1(bt, u);
+            Unit un = decode1(bt, ub);
+            for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
                 const int key = un.i * 65536 + un.s;
                 if (key != prev) {
@@ -370,8 +395,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
         const uint64_t cc = pack2(c, c);
         int64_t j = 0;                           // items of this group so far
         bool ok = true;
-        for (int64_t u = ub; u < ue && ok; ++u) {
-            const Unit un = decode1(bt, u);
+        Unit un = decode1(bt, ub);
+        for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
             const TcSender& sd = bt.s[un.i];
             const int halves = sd.R_pad / 128;
             const int64_t c0 = (int64_t)un.c * kChunk1;
@@ -526,8 +551,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             int64_t kt = 0, qn = 0;
             int prev = -1;
             bool ok = true;
-            for (int64_t u = ub; u < ue && ok; ++u) {
-                const Unit un = decode2(bt, u);
+            Unit un = decode2(bt, ub);
+            for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
                 const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
                 const int key = un.i * 65536 + un.s;
@@ -558,8 +583,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
             int prev = -1;
             bool ok = true;
-            for (int64_t u = ub; u < ue && ok; ++u) {
-                const Unit un = decode2(bt, u);
+            Unit un = decode2(bt, ub);
+            for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
                 const int key = un.i * 65536 + un.s;
                 if (key != prev) {
@@ -603,11 +628,13 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         int64_t j = 0, gt = 0;                   // chunks and tiles of this group so far
         int prev = -1;
         bool ok = true;
-        for (int64_t u = ub; u < ue && ok; ++u) {
-            const Unit un = decode2(bt, u);
+        float* part = nullptr;                   // U partials of the current group s
+        int64_t nST = 0;                         // distance between the U, N and D partials
+        Unit un = decode2(bt, ub);
+        if (grp == 1 && ub < ue) next2(bt, un);
+        for (int64_t u = ub + grp; u < ue && ok; u += 2, next2(bt, un), next2(bt, un)) {
             const TcSender& sd = bt.s[un.i];
             const int nch = (sd.R_pad + 255) / 256;
-            if (((u - ub) & 1) != grp) continue;
             const int key = un.i * 65536 + un.s;
             if (key != prev) {
                 __syncwarp();
@@ -617,6 +644,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 }
                 __syncwarp();
                 prev = key;
+                nST = (int64_t)bt.nL * bt.Hkv * sd.T;
+                part = sd.part + (int64_t)un.s * sd.T;
             }
             const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
             const bool valid = pos >= 0 && pos < sd.T;
@@ -660,13 +689,11 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 const float2 o = xs[lane];
                 nacc += o.x;
                 bsum += o.y;
-                const float inv_m = 1.f / (float)sd.m;
-                const float pb = lane_pool<PH>(bsum * inv_m);
+                const float pb = lane_pool<PH>(bsum * sd.inv_m);
                 if (valid && lane >= kMargin && lane < kMargin + kOutW) {
-                    const int64_t nS = (int64_t)bt.nL * bt.Hkv;
-                    sd.part[(0 * nS + un.s) * sd.T + pos] = bsum * inv_m / (float)bt.Hkv;
-                    sd.part[(1 * nS + un.s) * sd.T + pos] = nacc * inv_m;
-                    sd.part[(2 * nS + un.s) * sd.T + pos] = pow_p<P2>(pb, bt.p);
+                    part[pos] = bsum * sd.inv_mh;
+                    part[nST + pos] = nacc * sd.inv_m;
+                    part[2 * nST + pos] = pow_p<P2>(pb, bt.p);
                 }
             }
             ++gt;
@@ -773,6 +800,8 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             TcSender& d = tb->s[k];
             d.T = s.T;
             d.m = s.m;
+            d.inv_m = 1.f / (float)s.m;
+            d.inv_mh = 1.f / ((float)s.m * (float)b.n_kv_heads);
             d.R = s.m * G;
             d.R_pad = (d.R + 127) / 128 * 128;
             rpad_max = rpad_max > d.R_pad ? rpad_max : d.R_pad;
