@@ -163,7 +163,6 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
     constexpr int GT = (G + 1) / 2;
     constexpr int NBS = 4;  // n8 blocks per online-softmax step
     extern __shared__ __align__(128) uint4 ksm[];
-    const int nS = bt.n_layers * bt.n_kv_heads;
     const int64_t blk = blockIdx.x;
     const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blk1_begin; });
     const ScoreSender& sd = bt.s[i];

@@ -49,6 +49,7 @@ constexpr int kOutW = 32 - 2 * kMargin;          // 26 output positions per pass
 constexpr int kOut2 = 4 * kOutW;                 // 104 output positions per pass-2 tile
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitNs = 1000000000ull;      // 1 s per wait
+constexpr uint32_t kPollNs = 1000000u;           // longest suspension of one poll (woken at completion)
 constexpr int kMaxTcSenders = 32;
 
 struct TcSender {
@@ -98,7 +99,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Ctl* ct
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = now_ns();
     for (uint32_t i = 1; i < (1u << 30); ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait_hint(bar, parity, kPollNs)) return true;
         if ((i & 63) == 0) {
             if (*reinterpret_cast<volatile int*>(&ctl->abort)) return false;
             if (now_ns() - t0 > kWaitNs) {
@@ -239,15 +240,6 @@ __device__ __forceinline__ void mma_k128(uint32_t d_tmem, uint32_t a_base, uint3
     }
 }
 
-__device__ __forceinline__ void online_merge(float& m, float& l, float mo, float lo) {
-    const float mn = fmaxf(m, mo);
-    if (mn == -INFINITY) return;
-    const float a = (m == -INFINITY) ? 0.f : l * ex2(m - mn);
-    const float b = (mo == -INFINITY) ? 0.f : lo * ex2(mo - mn);
-    m = mn;
-    l = a + b;
-}
-
 // One 32-column block of pass 1 for this lane's row: running offset m (log2 domain) and
 // sum of exp2(c z - m).  The first block sets m to its max; later blocks reuse m and are
 // redone with their own max only if their sum could leave fp32 range (rare).
@@ -259,28 +251,27 @@ __device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c,
     if (m == -INFINITY) m = max_tree1(v) * c;
     if (m == -INFINITY) return;
     uint64_t nm = pack2(-m, -m);
-    uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};   // exp2 results are summed as scalars (no pair packing)
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
         float a0, a1;
         unpack2(ffma2(pack2(v[2 * q], v[2 * q + 1]), cc, nm), a0, a1);
-        acc[q & 3] = fadd2(acc[q & 3], pack2(ex2(a0), ex2(a1)));
+        acc[(2 * q) & 3] += ex2(a0);
+        acc[(2 * q + 1) & 3] += ex2(a1);
     }
-    float x0, x1;
-    unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
-    float blk = x0 + x1;
+    float blk = (acc[0] + acc[1]) + (acc[2] + acc[3]);
     if (!(blk <= 0x1p64f)) {
         const float mn = fmaxf(m, max_tree1(v) * c);
         nm = pack2(-mn, -mn);
-        acc[0] = acc[1] = acc[2] = acc[3] = 0ull;
+        acc[0] = acc[1] = acc[2] = acc[3] = 0.f;
 #pragma unroll
         for (int q = 0; q < 16; ++q) {
             float a0, a1;
             unpack2(ffma2(pack2(v[2 * q], v[2 * q + 1]), cc, nm), a0, a1);
-            acc[q & 3] = fadd2(acc[q & 3], pack2(ex2(a0), ex2(a1)));
+            acc[(2 * q) & 3] += ex2(a0);
+            acc[(2 * q + 1) & 3] += ex2(a1);
         }
-        unpack2(fadd2(fadd2(acc[0], acc[1]), fadd2(acc[2], acc[3])), x0, x1);
-        blk = x0 + x1;
+        blk = (acc[0] + acc[1]) + (acc[2] + acc[3]);
         sum *= ex2(m - mn);
         m = mn;
     }
@@ -315,7 +306,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (elect_one()) {
-            int64_t kt = 0, qn = 0;
+            int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
+            int st = 0;               // ring slot of the next K tile and its phase parity
+            uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
             Unit un = decode1(bt, ub);
@@ -331,10 +324,11 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                 }
                 const int64_t c0 = (int64_t)un.c * kChunk1;
                 const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
-                for (int tile = 0; tile < nt; ++tile, ++kt) {
-                    const int st = (int)(kt % stages);
-                    if (!(ok = wait_bar(&ctl->k_empty[st], (uint32_t)(((kt / stages) & 1) ^ 1), ctl, bt.err, 1))) break;
+                for (int tile = 0; tile < nt; ++tile) {
+                    if (!(ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 1))) break;
                     load_k(sd, sm, st, l, g, (int32_t)(c0 + tile * kTileRows));
+                    ++kt;
+                    if (++st == stages) { st = 0; ph ^= 1u; }
                 }
             }
             // drain: every issued load must land before the CTA exits
@@ -345,7 +339,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (elect_one()) {
-            int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
+            int64_t qn = 0, jg0 = 0, jg1 = 0;   // Q loads consumed; items issued per epilogue group
+            int st = 0;                          // ring slot of the next K tile and its phase parity
+            uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
             Unit un = decode1(bt, ub);
@@ -362,9 +358,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                 const int halves = sd.R_pad / 128;
                 const int64_t c0 = (int64_t)un.c * kChunk1;
                 const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
-                for (int tile = 0; tile < nt && ok; ++tile, ++kt) {
-                    const int st = (int)(kt % stages);
-                    if (!(ok = wait_bar(&ctl->k_full[st], (uint32_t)((kt / stages) & 1), ctl, bt.err, 3))) break;
+                for (int tile = 0; tile < nt && ok; ++tile) {
+                    if (!(ok = wait_bar(&ctl->k_full[st], ph, ctl, bt.err, 3))) break;
                     tc_fence_after();
                     const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
                     const int grp = tile & 1;     // epilogue group that owns this tile
@@ -378,6 +373,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                         umma_commit(&ctl->t_full[buf]);
                     }
                     umma_commit(&ctl->k_empty[st]);
+                    if (++st == stages) { st = 0; ph ^= 1u; }
                 }
             }
             umma_commit(&ctl->drain);
@@ -480,7 +476,7 @@ __device__ __forceinline__ float pow_p(float x, float p) {
 // column, b = sum over the G heads of each token, then Pool over positions and the sums.
 template <int G, int PH, bool P2>
 __device__ __forceinline__ void accum_block(const float (&v)[32], const float* negoff, uint64_t cc, bool valid,
-                                            bool all_valid, float p, uint64_t (&nacc2)[2], uint64_t (&bsum2)[2]) {
+                                            bool all_valid, float p, float (&nacc)[2], float (&bsum)[2]) {
     const float4* of4 = reinterpret_cast<const float4*>(negoff);
     float e[32];
 #pragma unroll
@@ -500,28 +496,42 @@ __device__ __forceinline__ void accum_block(const float (&v)[32], const float* n
     for (int k = 0; k < NT; ++k) {
         if (G == 1) b[k] = e[k];
         if (G == 2) b[k] = e[2 * k] + e[2 * k + 1];
-        if (G == 4) {
-            float x0, x1;
-            unpack2(fadd2(pack2(e[4 * k], e[4 * k + 1]), pack2(e[4 * k + 2], e[4 * k + 3])), x0, x1);
-            b[k] = x0 + x1;
-        }
+        if (G == 4) b[k] = (e[4 * k] + e[4 * k + 1]) + (e[4 * k + 2] + e[4 * k + 3]);
     }
     if (!all_valid) {
 #pragma unroll
         for (int k = 0; k < NT; ++k) b[k] = valid ? b[k] : 0.f;
     }
 #pragma unroll
-    for (int k = 0; k < NT; k += 2) {
-        const float p0 = lane_pool<PH>(b[k]), p1 = lane_pool<PH>(b[k + 1]);
-        const int a = (k >> 1) & 1;
-        bsum2[a] = fadd2(bsum2[a], pack2(b[k], b[k + 1]));
-        if (P2) {
-            const uint64_t pp = pack2(p0, p1);
-            nacc2[a] = ffma2(pp, pp, nacc2[a]);
-        } else {
-            nacc2[a] = fadd2(nacc2[a], pack2(pow_p<false>(p0, p), pow_p<false>(p1, p)));
-        }
+    for (int k = 0; k < NT; ++k) {
+        const float pk = lane_pool<PH>(b[k]);
+        bsum[k & 1] += b[k];
+        if (P2) nacc[k & 1] = fmaf(pk, pk, nacc[k & 1]);
+        else nacc[k & 1] += pow_p<false>(pk, p);
     }
+}
+
+// Pass 2, G = 4: head sums b of the four tokens in 16 columns (exp2(c z - offset) summed
+// over each token's four heads).
+__device__ __forceinline__ void head_sums16(const float (&v)[16], const float* negoff, uint64_t cc, float& b0,
+                                            float& b1, float& b2, float& b3) {
+    const float4* of4 = reinterpret_cast<const float4*>(negoff);
+    float e[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const float4 o = of4[q];
+        float a0, a1, a2, a3;
+        unpack2(ffma2(pack2(v[4 * q], v[4 * q + 1]), cc, pack2(o.x, o.y)), a0, a1);
+        unpack2(ffma2(pack2(v[4 * q + 2], v[4 * q + 3]), cc, pack2(o.z, o.w)), a2, a3);
+        e[4 * q] = ex2(a0);
+        e[4 * q + 1] = ex2(a1);
+        e[4 * q + 2] = ex2(a2);
+        e[4 * q + 3] = ex2(a3);
+    }
+    b0 = (e[0] + e[1]) + (e[2] + e[3]);
+    b1 = (e[4] + e[5]) + (e[6] + e[7]);
+    b2 = (e[8] + e[9]) + (e[10] + e[11]);
+    b3 = (e[12] + e[13]) + (e[14] + e[15]);
 }
 
 // Epilogue: each warp owns 32 TMEM lanes = positions t0 + 26 w - 3 + lane (w = lane quarter);
@@ -548,7 +558,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
 
     if (warp == 0) {
         if (elect_one()) {
-            int64_t kt = 0, qn = 0;
+            int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
+            int st = 0;               // ring slot of the next K tile and its phase parity
+            uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
             Unit un = decode2(bt, ub);
@@ -562,8 +574,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     ++qn;
                     prev = key;
                 }
-                const int st = (int)(kt % stages);
-                if (!(ok = wait_bar(&ctl->k_empty[st], (uint32_t)(((kt / stages) & 1) ^ 1), ctl, bt.err, 9))) break;
+                if (!(ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 9))) break;
                 // four 32-row boxes: quarter w holds positions t0 + 26 w - 3 .. + 31
                 uint8_t* dst = sm.k + (size_t)st * kTileBytes;
                 mbar_arrive_expect_tx(&ctl->k_full[st], kTileBytes);
@@ -573,6 +584,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                         tma_load_4d(dst + kb * (kTileBytes / 2) + w * 32 * 128, &sd.kmap32, &ctl->k_full[st],
                                     64 * kb, t0 + kOutW * w - kMargin, g, l);
                 ++kt;
+                if (++st == stages) { st = 0; ph ^= 1u; }
             }
             for (int64_t k = kt - stages > 0 ? kt - stages : 0; k < kt; ++k)
                 drain_wait(&ctl->k_full[k % stages], (uint32_t)((k / stages) & 1));
@@ -580,7 +592,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         }
     } else if (warp == 1) {
         if (elect_one()) {
-            int64_t kt = 0, qn = 0, jg0 = 0, jg1 = 0;   // items issued per epilogue group
+            int64_t qn = 0, jg0 = 0, jg1 = 0;   // Q loads consumed; items issued per epilogue group
+            int st = 0;                          // ring slot of the next K tile and its phase parity
+            uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
             Unit un = decode2(bt, ub);
@@ -594,8 +608,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     ++qn;
                     prev = key;
                 }
-                const int st = (int)(kt % stages);
-                if (!(ok = wait_bar(&ctl->k_full[st], (uint32_t)((kt / stages) & 1), ctl, bt.err, 11))) break;
+                if (!(ok = wait_bar(&ctl->k_full[st], ph, ctl, bt.err, 11))) break;
                 tc_fence_after();
                 const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
                 const int nch = (sd.R_pad + 255) / 256;
@@ -611,7 +624,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     umma_commit(&ctl->t_full[2 * grp]);
                 }
                 umma_commit(&ctl->k_empty[st]);
-                ++kt;
+                if (++st == stages) { st = 0; ph ^= 1u; }
             }
             umma_commit(&ctl->drain);
             drain_wait(&ctl->drain, 0);
@@ -650,7 +663,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
             const bool valid = pos >= 0 && pos < sd.T;
             const bool all_valid = __all_sync(0xffffffffu, valid);
-            uint64_t nacc2[2] = {0ull, 0ull}, bsum2[2] = {0ull, 0ull};   // pairs of token partial sums
+            float nacc2[2] = {0.f, 0.f}, bsum2[2] = {0.f, 0.f};   // token partial sums (two chains)
             for (int ci = 0; ci < nch && ok; ++ci) {
                 if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
                 ++j;
@@ -658,24 +671,47 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 const int ncol = min(128, min(256, sd.R_pad - 256 * ci) - hf * 128);   // this half's columns
                 const uint32_t ta = tmem + lane_addr + grp * 256 + hf * 128;
                 const float* ofc = offs + ci * 128;
-                // 32-column steps; sixteen epilogue warps hide the TMEM load latency
+                if (G == 4 && ncol > 0) {   // R_pad is a multiple of 128: ncol is 0 or 128
+                    // head sums of the warp's 32 tokens first, then the buffer goes back to the MMA
+                    // while Pool and the token sums run from registers
+                    float b[32];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        float v[16];
+                        tmem_ld16(ta + 16 * k, v);
+                        tmem_wait_ld();
+                        head_sums16(v, ofc + 16 * k, cc, b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
+                    if (!all_valid) {
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) b[k] = valid ? b[k] : 0.f;
+                    }
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) {
+                        const float pk = lane_pool<PH>(b[k]);
+                        bsum2[k & 1] += b[k];
+                        if (P2) nacc2[k & 1] = fmaf(pk, pk, nacc2[k & 1]);
+                        else nacc2[k & 1] += pow_p<false>(pk, bt.p);
+                    }
+                } else {
+                    // 32-column steps; sixteen epilogue warps hide the TMEM load latency
 #pragma unroll 1
-                for (int col = 0; col < ncol; col += 32) {
-                    float v[32];
-                    tmem_ld32(ta + col, v);
-                    tmem_wait_ld();
-                    accum_block<G, PH, P2>(v, ofc + col, cc, valid, all_valid, bt.p, nacc2, bsum2);
+                    for (int col = 0; col < (G == 4 ? 0 : ncol); col += 32) {
+                        float v[32];
+                        tmem_ld32(ta + col, v);
+                        tmem_wait_ld();
+                        accum_block<G, PH, P2>(v, ofc + col, cc, valid, all_valid, bt.p, nacc2, bsum2);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
                 }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
             }
             if (!ok) break;
-            float nacc, bsum, t0_, t1_;
-            unpack2(fadd2(nacc2[0], nacc2[1]), t0_, t1_);
-            nacc = t0_ + t1_;
-            unpack2(fadd2(bsum2[0], bsum2[1]), t0_, t1_);
-            bsum = t0_ + t1_;
+            float nacc = nacc2[0] + nacc2[1], bsum = bsum2[0] + bsum2[1];
             // the two column halves of the group add up their sums; half 0 writes the results
             const int tp = (int)(gt & 1);
             float2* xs = xch + ((tp * 2 + grp) * 4 + sp) * 32;
