@@ -53,6 +53,8 @@ struct cb_ctx {
     int64_t n_chunk1_max = 0;
     float2* stats = nullptr;
     float* offs = nullptr;
+    uint16_t* ext = nullptr;        // tcgen05 passes: per-row offset terms [S][nS][R_pad][16] bf16
+    uint16_t* ones = nullptr;       // tcgen05 passes: [128][16] bf16 block of ones columns
     float* part = nullptr;
     float* fin = nullptr;
     float* span_keys = nullptr;
@@ -217,6 +219,16 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     if (e == cudaSuccess) e = alloc(&ctx->part, (size_t)(S * 3 * nS * c.max_positions), &total);
     if (e == cudaSuccess) e = alloc(&ctx->fin, (size_t)(S * cbk::kFinSlices * 3 * c.max_positions), &total);
     if (e == cudaSuccess) e = alloc(&ctx->span_keys, (size_t)(S * ctx->keys_per_sender), &total);
+    if (e == cudaSuccess && ctx->use_tc) {
+        e = alloc(&ctx->ext, (size_t)(S * nS * cbk::rows_pad128(rows) * cbk::kExtCols), &total);
+        if (e == cudaSuccess) e = alloc(&ctx->ones, (size_t)(128 * cbk::kExtCols), &total);
+        if (e == cudaSuccess) {
+            std::vector<uint16_t> h(128 * cbk::kExtCols, 0);
+            for (int r = 0; r < 128; ++r)
+                for (int k = 0; k < 3; ++k) h[r * cbk::kExtCols + k] = 0x3F80;   // bf16 1.0
+            e = cudaMemcpy(ctx->ones, h.data(), h.size() * sizeof(uint16_t), cudaMemcpyHostToDevice);
+        }
+    }
     if (e == cudaSuccess) e = alloc(&ctx->err, 1, &total);
     if (e == cudaSuccess) e = cudaMemset(ctx->err, 0, sizeof(uint32_t));
     ctx->scratch_bytes = total;
@@ -237,6 +249,8 @@ void cb_destroy(cb_ctx* ctx) {
         cudaDeviceSynchronize();
         cudaFree(ctx->stats);
         cudaFree(ctx->offs);
+        cudaFree(ctx->ext);
+        cudaFree(ctx->ones);
         cudaFree(ctx->part);
         cudaFree(ctx->fin);
         cudaFree(ctx->span_keys);
@@ -291,9 +305,11 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->err = ctx->err;
         bt->stats = ctx->stats;
         bt->offs = ctx->offs;
+        bt->ext = ctx->use_tc ? ctx->ext : nullptr;
+        bt->ones = ctx->ones;
         bt->part = ctx->part;
         bt->fin = ctx->fin;
-        int64_t so = 0, oo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
+        int64_t so = 0, oo = 0, eo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
             const cb_query& q = queries[b0 + k];
@@ -309,6 +325,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.n_chunk2 = (int32_t)((s.T + cbk::kAccumChunk - 1) / cbk::kAccumChunk);
             d.stats_off = so; so += (int64_t)nS * cbk::stats_slots(s.T) * q.m * ctx->G;
             d.offs_off = oo; oo += (int64_t)nS * q.m * ctx->G;
+            d.ext_off = eo; eo += (int64_t)nS * cbk::rows_pad128((int64_t)q.m * ctx->G) * cbk::kExtCols;
             d.part_off = po; po += (int64_t)3 * nS * s.T;
             d.fin_off = fo; fo += (int64_t)cbk::kFinSlices * 3 * s.T;
             d.blk1_begin = b1; b1 += (int64_t)nS * d.n_chunk1;

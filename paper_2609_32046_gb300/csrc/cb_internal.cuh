@@ -47,6 +47,7 @@ struct ScoreSender {
     int32_t n_chunk2;         // ceil(T / kAccumChunk)
     int64_t stats_off;        // float2 offset of this sender's pass-1 partials
     int64_t offs_off;         // float offset of this sender's per-row softmax offsets
+    int64_t ext_off;          // bf16 offset of this sender's [nS][R_pad][16] offset rows (tcgen05 passes)
     int64_t part_off;         // float offset of this sender's [3][nS][T] partials
     int64_t fin_off;          // float offset of this sender's [kFinSlices][3][T] slice sums
     int64_t blk1_begin;       // first pass-1 block of this sender
@@ -65,10 +66,18 @@ struct ScoreBatch {
     StageTimer* timer;        // host-side; null unless stage timing is enabled
     float2* stats;            // pass-1 partial (max, sum) in log2 domain
     float* offs;              // per-row log2 offsets (max + log2(sum) + log2(G))
+    uint16_t* ext;            // tcgen05 passes: -offset / scale_log2e per row as three bf16 terms
+                              // (hi, mid, lo, then 13 zeros; -1e30 on padding rows), else null
+    const uint16_t* ones;     // tcgen05 passes: [128][16] bf16, columns 0-2 = 1, the rest 0
     float* part;              // per-group U_s, N_s, D_s partials
     float* fin;               // finalize slice sums [sender][kFinSlices][3][T]
     ScoreSender s[kMaxBatch];
 };
+
+constexpr int kExtCols = 16;   // one bf16 K-step: the extra contraction column block of pass 2
+
+// Query rows padded to the 128-row granule of the tcgen05 passes.
+__host__ __device__ inline int64_t rows_pad128(int64_t rows) { return (rows + 127) / 128 * 128; }
 
 struct SelectSender {
     const float* scores;

@@ -16,6 +16,7 @@
 // normaliser over all T positions, pass 2 recomputes the logits and normalises.
 #include <cfloat>
 #include <cstdint>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "cb_internal.cuh"
@@ -248,18 +249,42 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
     const ScoreSender& sd = bt.s[i];
     const int R = sd.m * G;
     const float lg = log2f((float)G);
-    for (int row = threadIdx.x; row < R; row += kThreads) {
-        const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
-        float M = -INFINITY;
+    const int R_pad = (int)rows_pad128(R);
+    for (int row = threadIdx.x; row < (bt.ext ? R_pad : R); row += kThreads) {
+        float off = 0.f;
+        if (row < R) {
+            const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
+            float M = -INFINITY;
 #pragma unroll 8
-        for (int c = 0; c < sd.n_chunk1; ++c) M = fmaxf(M, st[(int64_t)c * R].x);
-        float L = 0.f;
+            for (int c = 0; c < sd.n_chunk1; ++c) M = fmaxf(M, st[(int64_t)c * R].x);
+            float L = 0.f;
 #pragma unroll 8
-        for (int c = 0; c < sd.n_chunk1; ++c) {
-            const float2 v = st[(int64_t)c * R];
-            if (v.x != -INFINITY) L += v.y * ex2(v.x - M);
+            for (int c = 0; c < sd.n_chunk1; ++c) {
+                const float2 v = st[(int64_t)c * R];
+                if (v.x != -INFINITY) L += v.y * ex2(v.x - M);
+            }
+            off = M + log2f(L) + lg;
+            bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
         }
-        bt.offs[sd.offs_off + (int64_t)s * R + row] = M + log2f(L) + lg;
+        if (bt.ext) {
+            // the tcgen05 pass 2 adds -off / scale_log2e to the logit inside the contraction
+            // (one more K-step against a column of ones): three bf16 terms carry it to ~24 bits
+            uint32_t w0 = 0, w1 = 0;
+            if (row < R) {
+                const float x = -off / bt.scale_log2e;
+                const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+                const float r1 = x - __bfloat162float(hi);
+                const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+                const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+                w0 = (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(mid) << 16);
+                w1 = (uint32_t)__bfloat16_as_ushort(lo);
+            } else {
+                w0 = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(-1e30f));   // exp2 of it is 0
+            }
+            uint4* dst = reinterpret_cast<uint4*>(bt.ext + sd.ext_off + ((int64_t)s * R_pad + row) * kExtCols);
+            dst[0] = make_uint4(w0, w1, 0u, 0u);
+            dst[1] = make_uint4(0u, 0u, 0u, 0u);
+        }
     }
 }
 

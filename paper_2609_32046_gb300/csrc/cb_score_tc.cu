@@ -56,6 +56,7 @@ struct TcSender {
     CUtensorMap kmap;     // 4D {d, T, Hkv, nL}, box {64, 128, 1, 1}
     CUtensorMap kmap32;   // same tensor, box {64, 32, 1, 1}
     CUtensorMap qmap;     // 4D {d, Hq, m, nL}, box {64, G, qbox_tok, 1}
+    CUtensorMap emap;     // 3D {16, R_pad, nS} offset terms of pass 2, box {16, ebox_rows, 1}, 32-byte swizzle
     float2* stats;        // this sender's pass-1 partials [nS][n_chunk1][R]
     const float* offs;    // this sender's per-row offsets [nS][R]
     float* part;          // this sender's partials [3][nS][T]
@@ -63,11 +64,13 @@ struct TcSender {
     int32_t m, R, R_pad;
     int32_t n_chunk1, n_tile2;
     int32_t qbox_tok, n_qbox;
+    int32_t ebox_rows, n_ebox;
     float inv_m, inv_mh;  // 1 / m and 1 / (m Hkv)
     int64_t unit1_begin, unit2_begin;
 };
 
 struct TcBatch {
+    CUtensorMap omap;     // 2D {16, 128} block of ones columns, one box, 32-byte swizzle
     int32_t n;
     int32_t nL, Hq, Hkv, G;
     int32_t stages, rpad_max;
@@ -81,7 +84,7 @@ struct TcBatch {
 struct Ctl {
     uint64_t k_full[kMaxStages], k_empty[kMaxStages];
     uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns; group g owns 2g and 2g + 1
-    uint64_t q_full, q_empty, drain;
+    uint64_t q_full, q_empty, drain, o_full;
     uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]
     uint32_t tmem_base;
     int abort;
@@ -174,9 +177,12 @@ __device__ __forceinline__ void my_range(int64_t total, int64_t* b, int64_t* e) 
     *e = total * (blockIdx.x + 1) / gridDim.x;
 }
 
-// Shared memory: [Q: 2 blocks x rpad x 128 B][K ring: stages x 32 KB][Ctl][epilogue scratch]
+// Shared memory: [Q: 2 blocks x rpad x 128 B][offset terms: rpad x 32 B][ones: 4 KB]
+// [K ring: stages x 32 KB][Ctl][epilogue scratch]
 struct Smem {
     uint8_t* q;
+    uint8_t* ext;     // pass 2: offset terms of Q's rows [rpad][32 B], 32-byte swizzle
+    uint8_t* ones;    // pass 2: ones columns [128][32 B], 32-byte swizzle
     uint8_t* k;
     Ctl* ctl;
     float* epi;
@@ -186,7 +192,9 @@ __device__ __forceinline__ Smem carve(uint8_t* raw, const TcBatch& bt) {
     Smem sm;
     uint8_t* base = align1024(raw);
     sm.q = base;
-    sm.k = base + (size_t)2 * bt.rpad_max * 128;
+    sm.ext = base + (size_t)2 * bt.rpad_max * 128;
+    sm.ones = sm.ext + (size_t)bt.rpad_max * 32;
+    sm.k = sm.ones + 128 * 32;
     sm.ctl = reinterpret_cast<Ctl*>(sm.k + (size_t)bt.stages * kTileBytes);
     sm.epi = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sm.ctl) + 512);
     return sm;
@@ -204,15 +212,22 @@ __device__ __forceinline__ void init_ctl(Ctl* ctl, int stages) {
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
     mbar_init(&ctl->drain, 1);
+    mbar_init(&ctl->o_full, 1);
     for (int k = 0; k < 16; ++k) mbar_init(&ctl->xb[k >> 3][(k >> 2) & 1][k & 3], 1);
     ctl->abort = 0;
     fence_barrier_init();
 }
 
 // Producer: Q of group s (all rows, both column blocks) into the Q region.
-__device__ __forceinline__ void load_q(const TcBatch& bt, const TcSender& sd, const Smem& sm, int l, int g) {
-    const uint32_t bytes = (uint32_t)sd.R_pad * 256u;
+// Pass 2 (with_ext) also brings the rows' offset terms of group s = l * Hkv + g.
+__device__ __forceinline__ void load_q(const TcBatch& bt, const TcSender& sd, const Smem& sm, int l, int g,
+                                       bool with_ext) {
+    const uint32_t bytes = (uint32_t)sd.R_pad * (with_ext ? 256u + 32u : 256u);
     mbar_arrive_expect_tx(&sm.ctl->q_full, bytes);
+    if (with_ext)
+        for (int b = 0; b < sd.n_ebox; ++b)
+            tma_load_3d(sm.ext + (size_t)b * sd.ebox_rows * 32, &sd.emap, &sm.ctl->q_full, 0, b * sd.ebox_rows,
+                        l * bt.Hkv + g);
     for (int kb = 0; kb < 2; ++kb)
         for (int b = 0; b < sd.n_qbox; ++b)
             tma_load_4d(sm.q + (size_t)kb * bt.rpad_max * 128 + (size_t)b * sd.qbox_tok * bt.G * 128, &sd.qmap,
@@ -318,7 +333,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                 const int key = un.i * 65536 + un.s;
                 if (key != prev) {
                     if (!(ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 0))) break;
-                    load_q(bt, sd, sm, l, g);
+                    load_q(bt, sd, sm, l, g, false);
                     ++qn;
                     prev = key;
                 }
@@ -475,16 +490,14 @@ __device__ __forceinline__ float pow_p(float x, float p) {
 // One 32-column block of pass 2 for this lane's position: a / G = exp2(c z - offset) per
 // column, b = sum over the G heads of each token, then Pool over positions and the sums.
 template <int G, int PH, bool P2>
-__device__ __forceinline__ void accum_block(const float (&v)[32], const float* negoff, uint64_t cc, bool valid,
-                                            bool all_valid, float p, float (&nacc)[2], float (&bsum)[2]) {
-    const float4* of4 = reinterpret_cast<const float4*>(negoff);
+__device__ __forceinline__ void accum_block(const float (&v)[32], uint64_t cc, bool valid, bool all_valid, float p,
+                                            float (&nacc)[2], float (&bsum)[2]) {
     float e[32];
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-        const float4 o = of4[q];
         float a0, a1, a2, a3;
-        unpack2(ffma2(pack2(v[4 * q], v[4 * q + 1]), cc, pack2(o.x, o.y)), a0, a1);
-        unpack2(ffma2(pack2(v[4 * q + 2], v[4 * q + 3]), cc, pack2(o.z, o.w)), a2, a3);
+        unpack2(fmul2(pack2(v[4 * q], v[4 * q + 1]), cc), a0, a1);
+        unpack2(fmul2(pack2(v[4 * q + 2], v[4 * q + 3]), cc), a2, a3);
         e[4 * q] = ex2(a0);
         e[4 * q + 1] = ex2(a1);
         e[4 * q + 2] = ex2(a2);
@@ -513,16 +526,14 @@ __device__ __forceinline__ void accum_block(const float (&v)[32], const float* n
 
 // Pass 2, G = 4: head sums b of the four tokens in 16 columns (exp2(c z - offset) summed
 // over each token's four heads).
-__device__ __forceinline__ void head_sums16(const float (&v)[16], const float* negoff, uint64_t cc, float& b0,
-                                            float& b1, float& b2, float& b3) {
-    const float4* of4 = reinterpret_cast<const float4*>(negoff);
+__device__ __forceinline__ void head_sums16(const float (&v)[16], uint64_t cc, float& b0, float& b1, float& b2,
+                                            float& b3) {
     float e[16];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        const float4 o = of4[q];
         float a0, a1, a2, a3;
-        unpack2(ffma2(pack2(v[4 * q], v[4 * q + 1]), cc, pack2(o.x, o.y)), a0, a1);
-        unpack2(ffma2(pack2(v[4 * q + 2], v[4 * q + 3]), cc, pack2(o.z, o.w)), a2, a3);
+        unpack2(fmul2(pack2(v[4 * q], v[4 * q + 1]), cc), a0, a1);
+        unpack2(fmul2(pack2(v[4 * q + 2], v[4 * q + 3]), cc), a2, a3);
         e[4 * q] = ex2(a0);
         e[4 * q + 1] = ex2(a1);
         e[4 * q + 2] = ex2(a2);
@@ -563,6 +574,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
+            // the ones columns of the offset K-step, once per CTA
+            mbar_arrive_expect_tx(&ctl->o_full, 128 * 32);
+            tma_load_2d(sm.ones, &bt.omap, &ctl->o_full, 0, 0);
             Unit un = decode2(bt, ub);
             for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
@@ -570,7 +584,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 const int key = un.i * 65536 + un.s;
                 if (key != prev) {
                     if (!(ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 8))) break;
-                    load_q(bt, sd, sm, l, g);
+                    load_q(bt, sd, sm, l, g, true);
                     ++qn;
                     prev = key;
                 }
@@ -589,6 +603,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             for (int64_t k = kt - stages > 0 ? kt - stages : 0; k < kt; ++k)
                 drain_wait(&ctl->k_full[k % stages], (uint32_t)((k / stages) & 1));
             if (qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
+            drain_wait(&ctl->o_full, 0);
         }
     } else if (warp == 1) {
         if (elect_one()) {
@@ -596,7 +611,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             int st = 0;                          // ring slot of the next K tile and its phase parity
             uint32_t ph = 0;
             int prev = -1;
-            bool ok = true;
+            bool ok = wait_bar(&ctl->o_full, 0, ctl, bt.err, 15);
+            tc_fence_after();
+            const uint64_t ones_desc = smem_desc_sw32(smem_u32(sm.ones));
+            const uint64_t ext_desc = smem_desc_sw32(smem_u32(sm.ext));
             Unit un = decode2(bt, ub);
             for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
@@ -621,6 +639,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     const int ncol = min(256, sd.R_pad - 256 * c);
                     mma_k128(tmem + grp * 256, kaddr, kTileBytes / 2, smem_u32(sm.q) + c * 256 * 128,
                              (uint32_t)bt.rpad_max * 128, idesc_bf16_f32(128, ncol));
+                    // one more K-step: ones (positions) x offset terms (rows) adds -offset / scale to
+                    // every logit, so the epilogue needs only exp2(scale * D)
+                    umma_bf16(tmem + grp * 256, ones_desc, ext_desc + (uint64_t)((c * 256 * 32) >> 4),
+                              idesc_bf16_f32(128, ncol), 1u);
                     umma_commit(&ctl->t_full[2 * grp]);
                 }
                 umma_commit(&ctl->k_empty[st]);
@@ -634,43 +656,56 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         // takes columns half*128 .. +128 of each 256-column chunk (32 tokens when G = 4).
         const int ew = warp - 2, quad = ew >> 2, grp = quad >> 1, hf = quad & 1, sp = warp & 3;
         const uint32_t lane_addr = (uint32_t)(sp * 32) << 16;
-        float* offs = sm.epi + ew * 256;          // this warp's negated row offsets: [chunk][128]
-        float2* xch = reinterpret_cast<float2*>(sm.epi + 16 * 256);   // [parity][grp][sp][32]
+        float2* xch = reinterpret_cast<float2*>(sm.epi);   // [parity][grp][sp][32]
         const float c = bt.sl2e;
         const uint64_t cc = pack2(c, c);
         int64_t j = 0, gt = 0;                   // chunks and tiles of this group so far
         int prev = -1;
         bool ok = true;
+        // per-sender values live in registers and are refreshed when the group s changes
+        // (indexed reads of the kernel-parameter block on every tile are slow)
         float* part = nullptr;                   // U partials of the current group s
         int64_t nST = 0;                         // distance between the U, N and D partials
+        int64_t T = 0;
+        int nch = 0, n_tile = 1, R_pad = 0;
+        float inv_m = 0.f, inv_mh = 0.f;
+        const int nS = bt.nL * bt.Hkv;
         Unit un = decode2(bt, ub);
-        if (grp == 1 && ub < ue) next2(bt, un);
-        for (int64_t u = ub + grp; u < ue && ok; u += 2, next2(bt, un), next2(bt, un)) {
-            const TcSender& sd = bt.s[un.i];
-            const int nch = (sd.R_pad + 255) / 256;
+        n_tile = bt.s[un.i].n_tile2;
+        auto advance = [&]() {   // next unit (sender, group, tile) without parameter reads
+            if (++un.c == n_tile) {
+                un.c = 0;
+                if (++un.s == nS) {
+                    un.s = 0;
+                    ++un.i;
+                    if (un.i < bt.n) n_tile = bt.s[un.i].n_tile2;
+                }
+            }
+        };
+        if (grp == 1 && ub < ue) advance();
+        for (int64_t u = ub + grp; u < ue && ok; u += 2, advance(), advance()) {
             const int key = un.i * 65536 + un.s;
             if (key != prev) {
-                __syncwarp();
-                for (int k = lane; k < nch * 128; k += 32) {
-                    const int r = (k >> 7) * 256 + hf * 128 + (k & 127);
-                    offs[k] = r < sd.R ? -sd.offs[(int64_t)un.s * sd.R + r] : -INFINITY;
-                }
-                __syncwarp();
-                prev = key;
-                nST = (int64_t)bt.nL * bt.Hkv * sd.T;
+                const TcSender& sd = bt.s[un.i];
+                R_pad = sd.R_pad;
+                nch = (sd.R_pad + 255) / 256;
+                T = sd.T;
+                inv_m = sd.inv_m;
+                inv_mh = sd.inv_mh;
+                nST = (int64_t)nS * sd.T;
                 part = sd.part + (int64_t)un.s * sd.T;
+                prev = key;
             }
             const int64_t pos = (int64_t)un.c * kOut2 + kOutW * sp - kMargin + lane;
-            const bool valid = pos >= 0 && pos < sd.T;
+            const bool valid = pos >= 0 && pos < T;
             const bool all_valid = __all_sync(0xffffffffu, valid);
             float nacc2[2] = {0.f, 0.f}, bsum2[2] = {0.f, 0.f};   // token partial sums (two chains)
             for (int ci = 0; ci < nch && ok; ++ci) {
                 if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
                 ++j;
                 tc_fence_after();
-                const int ncol = min(128, min(256, sd.R_pad - 256 * ci) - hf * 128);   // this half's columns
+                const int ncol = min(128, min(256, R_pad - 256 * ci) - hf * 128);   // this half's columns
                 const uint32_t ta = tmem + lane_addr + grp * 256 + hf * 128;
-                const float* ofc = offs + ci * 128;
                 if (G == 4 && ncol > 0) {   // R_pad is a multiple of 128: ncol is 0 or 128
                     // head sums of the warp's 32 tokens first, then the buffer goes back to the MMA
                     // while Pool and the token sums run from registers
@@ -679,8 +714,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     for (int k = 0; k < 8; ++k) {
                         float v[16];
                         tmem_ld16(ta + 16 * k, v);
-                        tmem_wait_ld();
-                        head_sums16(v, ofc + 16 * k, cc, b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
+                        tmem_wait_ld(v);
+                        head_sums16(v, cc, b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -703,7 +738,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                         float v[32];
                         tmem_ld32(ta + col, v);
                         tmem_wait_ld();
-                        accum_block<G, PH, P2>(v, ofc + col, cc, valid, all_valid, bt.p, nacc2, bsum2);
+                        accum_block<G, PH, P2>(v, cc, valid, all_valid, bt.p, nacc2, bsum2);
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -725,10 +760,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 const float2 o = xs[lane];
                 nacc += o.x;
                 bsum += o.y;
-                const float pb = lane_pool<PH>(bsum * sd.inv_m);
+                const float pb = lane_pool<PH>(bsum * inv_m);
                 if (valid && lane >= kMargin && lane < kMargin + kOutW) {
-                    part[pos] = bsum * sd.inv_mh;
-                    part[nST + pos] = nacc * sd.inv_m;
+                    part[pos] = bsum * inv_mh;
+                    part[nST + pos] = nacc * inv_m;
                     part[2 * nST + pos] = pow_p<P2>(pb, bt.p);
                 }
             }
@@ -760,18 +795,25 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
     return g_encode;
 }
 
-bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4], const cuuint64_t strides_bytes[3],
-               const cuuint32_t box[4]) {
+// bf16 tensor map of `rank` dimensions (innermost first); strides in bytes of dims 1..rank-1.
+bool encode_nd(CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims, const cuuint64_t* strides_bytes,
+               const cuuint32_t* box, CUtensorMapSwizzle swizzle) {
     auto fn = encoder();
-    if (!fn) return false;
+    if (!fn || !base) return false;
     const cuuint32_t es[4] = {1, 1, 1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides_bytes, box, es,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims, strides_bytes, box,
+              es, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4], const cuuint64_t strides_bytes[3],
+               const cuuint32_t box[4]) {
+    return encode_nd(m, base, 4, dims, strides_bytes, box, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
 size_t smem_bytes(int rpad_max, int stages) {
-    return 1024 + (size_t)2 * rpad_max * 128 + (size_t)stages * kTileBytes + 512 + 16 * 256 * 4 + 2 * 2 * 4 * 32 * 8;
+    return 1024 + (size_t)2 * rpad_max * 128 + (size_t)rpad_max * 32 + 128 * 32 + (size_t)stages * kTileBytes + 512 +
+           2 * 2 * 4 * 32 * 8;
 }
 
 template <int G, int PH, bool P2>
@@ -866,11 +908,25 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             const cuuint64_t qs[3] = {(cuuint64_t)s.qs_h * 2, (cuuint64_t)s.qs_t * 2, (cuuint64_t)s.qs_l * 2};
             const cuuint32_t qbox[4] = {64, (cuuint32_t)G, (cuuint32_t)d.qbox_tok, 1};
             const cuuint32_t kbox32[4] = {64, 32, 1, 1};
+            // offset terms [nS][R_pad][16] written by the combine kernel, boxes of at most 256 rows
+            d.ebox_rows = d.R_pad <= 256 ? d.R_pad : 128;
+            d.n_ebox = d.R_pad / d.ebox_rows;
+            const cuuint64_t ed[3] = {(cuuint64_t)kExtCols, (cuuint64_t)d.R_pad, (cuuint64_t)nS};
+            const cuuint64_t es[2] = {(cuuint64_t)kExtCols * 2, (cuuint64_t)d.R_pad * kExtCols * 2};
+            const cuuint32_t ebox[3] = {(cuuint32_t)kExtCols, (cuuint32_t)d.ebox_rows, 1};
             if (!encode_4d(&d.kmap, s.k, kd, ks, kbox) || !encode_4d(&d.kmap32, s.k, kd, ks, kbox32) ||
-                !encode_4d(&d.qmap, s.q, qd, qs, qbox)) {
+                !encode_4d(&d.qmap, s.q, qd, qs, qbox) || d.n_ebox * d.ebox_rows != d.R_pad || !b.ext ||
+                !encode_nd(&d.emap, b.ext + s.ext_off, 3, ed, es, ebox, CU_TENSOR_MAP_SWIZZLE_32B)) {
                 free_all();
                 return cudaErrorNotSupported;
             }
+        }
+        const cuuint64_t od[2] = {(cuuint64_t)kExtCols, 128};
+        const cuuint64_t os[1] = {(cuuint64_t)kExtCols * 2};
+        const cuuint32_t obox[2] = {(cuuint32_t)kExtCols, 128};
+        if (!encode_nd(&tb->omap, b.ones, 2, od, os, obox, CU_TENSOR_MAP_SWIZZLE_32B)) {
+            free_all();
+            return cudaErrorNotSupported;
         }
         tb->rpad_max = rpad_max;
         tb->stages = rpad_max > 256 ? 2 : 4;
