@@ -185,6 +185,12 @@ const char *cb_last_error(const cb_ctx *ctx);
 /* Device scratch bytes the context holds (for capacity planning). */
 int64_t cb_scratch_bytes(const cb_ctx *ctx);
 
+/* Which implementation of the two logit passes (App. C.1) the context's last cb_score launched:
+ * 2 = tcgen05 (tensor-memory) kernels, 1 = mma.sync kernels, 0 = no cb_score yet or NULL ctx.
+ * With score_kernel = 0 or 2 the tcgen05 kernels run unless the driver rejects a tensor map for
+ * the given strides; then the mma.sync kernels run instead and this reports 1.  Host-only. */
+int32_t cb_score_path(const cb_ctx *ctx);
+
 /*
  * Allocation-free selection.  The paper has no counterpart: this entry point exists
  * for callers that cannot allocate device memory (code running inside a memory pool or

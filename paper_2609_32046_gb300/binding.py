@@ -20,7 +20,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
-            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_select_noalloc",
+            "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
             "cb_enable_stage_timing", "cb_stage_times"]
 
 
@@ -85,6 +85,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_last_error.restype = ctypes.c_char_p
     lib.cb_scratch_bytes.argtypes = [P]
     lib.cb_scratch_bytes.restype = ctypes.c_int64
+    lib.cb_score_path.argtypes = [P]
+    lib.cb_score_path.restype = ctypes.c_int32
     lib.cb_select_noalloc.argtypes = [ctypes.c_int32, P, P, P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
     lib.cb_select_noalloc.restype = ctypes.c_int
     lib.cb_enable_stage_timing.argtypes = [P, ctypes.c_int32]
@@ -184,6 +186,10 @@ class CacheBack:
     @property
     def scratch_bytes(self) -> int:
         return int(self.lib.cb_scratch_bytes(self.h))
+
+    def score_path(self) -> int:
+        """Logit-pass kernels of the last score call: 2 tcgen05, 1 mma.sync, 0 none yet."""
+        return int(self.lib.cb_score_path(self.h))
 
     # -- the three steps ----------------------------------------------------
     def score(self, Ks: Sequence, Qs: Sequence, scores: Sequence, stream=None):

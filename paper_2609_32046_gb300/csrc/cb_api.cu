@@ -61,6 +61,7 @@ struct cb_ctx {
     uint32_t* err = nullptr;
     int64_t keys_per_sender = 0;
     int64_t scratch_bytes = 0;
+    int32_t score_path = 0;         // kernels of the last cb_score: 2 tcgen05, 1 mma.sync, 0 none yet
     cbk::StageTimer* timer = nullptr;
     std::string last_error;
 };
@@ -159,6 +160,8 @@ int64_t cb_budget(int64_t T, double keep) {
 const char* cb_last_error(const cb_ctx* ctx) { return ctx ? ctx->last_error.c_str() : g_create_error.c_str(); }
 
 int64_t cb_scratch_bytes(const cb_ctx* ctx) { return ctx ? ctx->scratch_bytes : 0; }
+
+int32_t cb_score_path(const cb_ctx* ctx) { return ctx ? ctx->score_path : 0; }
 
 cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     if (!out) return fail(nullptr, CB_EINVAL, "out is NULL");
@@ -332,7 +335,9 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
             d.blkf_begin = 0;  // set by the score launcher
         }
-        cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms);
+        int path = 0;
+        cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms, &path);
+        ctx->score_path = path;
         delete bt;
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "score launch failed: %s", cudaGetErrorString(e));
     }

@@ -123,7 +123,8 @@ void set_context_free_error(const char* msg);
 bool tc_path_supported(int head_dim, int G, int pool_half, int max_query_tokens);
 
 // Launchers (return the launch error, if any).
-cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms);
+// *path_out: 2 when the tcgen05 passes ran, 1 for the mma.sync passes.
+cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms, int* path_out);
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);
 cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms);
 

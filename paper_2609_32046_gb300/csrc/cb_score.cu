@@ -243,48 +243,83 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // combine: per-row log2 offset = max + log2(sum) + log2(G) over all chunks
 // ---------------------------------------------------------------------------
+// Block = 64 rows x 4 slot lanes of one (sender, group s): slot lane j merges partial slots
+// j, j + 4, ... of its row with an online max/sum, then slot lane 0 merges the four results
+// in lane order (a fixed order, so the offsets are deterministic).
+constexpr int kCombRows = 64;
 __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
+    __shared__ float2 part[4][kCombRows];
     const int nS = bt.n_layers * bt.n_kv_heads;
-    const int i = blockIdx.x / nS, s = blockIdx.x % nS;
-    const ScoreSender& sd = bt.s[i];
+    const ScoreSender* sdp = nullptr;
+    int i = 0;
+    int64_t blk = blockIdx.x;
+    // blocks are laid out sender by sender, nS * ceil(R_pad / 64) of them per sender
+    for (; i < bt.n; ++i) {
+        const int R_i = bt.s[i].m * G;
+        const int rows_i = bt.ext ? (int)rows_pad128(R_i) : R_i;
+        const int64_t nb = (int64_t)nS * ((rows_i + kCombRows - 1) / kCombRows);
+        if (blk < nb) break;
+        blk -= nb;
+    }
+    if (i >= bt.n) return;
+    sdp = &bt.s[i];
+    const ScoreSender& sd = *sdp;
     const int R = sd.m * G;
-    const float lg = log2f((float)G);
-    const int R_pad = (int)rows_pad128(R);
-    for (int row = threadIdx.x; row < (bt.ext ? R_pad : R); row += kThreads) {
-        float off = 0.f;
-        if (row < R) {
-            const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
-            float M = -INFINITY;
-#pragma unroll 8
-            for (int c = 0; c < sd.n_chunk1; ++c) M = fmaxf(M, st[(int64_t)c * R].x);
-            float L = 0.f;
-#pragma unroll 8
-            for (int c = 0; c < sd.n_chunk1; ++c) {
-                const float2 v = st[(int64_t)c * R];
-                if (v.x != -INFINITY) L += v.y * ex2(v.x - M);
-            }
-            off = M + log2f(L) + lg;
-            bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
-        }
-        if (bt.ext) {
-            // the tcgen05 pass 2 adds -off / scale_log2e to the logit inside the contraction
-            // (one more K-step against a column of ones): three bf16 terms carry it to ~24 bits
-            uint32_t w0 = 0, w1 = 0;
-            if (row < R) {
-                const float x = -off / bt.scale_log2e;
-                const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-                const float r1 = x - __bfloat162float(hi);
-                const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
-                const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
-                w0 = (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(mid) << 16);
-                w1 = (uint32_t)__bfloat16_as_ushort(lo);
+    const int rows = bt.ext ? (int)rows_pad128(R) : R;
+    const int nrb = (rows + kCombRows - 1) / kCombRows;
+    const int s = (int)(blk / nrb);
+    const int row = (int)(blk % nrb) * kCombRows + (threadIdx.x & (kCombRows - 1));
+    const int j = threadIdx.x / kCombRows;   // slot lane 0..3
+    float M = -INFINITY, L = 0.f;
+    if (row < R) {
+        const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
+#pragma unroll 4
+        for (int c = j; c < sd.n_chunk1; c += 4) {
+            const float2 v = st[(int64_t)c * R];
+            if (v.x == -INFINITY) continue;
+            if (v.x > M) {
+                L = (M == -INFINITY ? 0.f : L * ex2(M - v.x)) + v.y;
+                M = v.x;
             } else {
-                w0 = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(-1e30f));   // exp2 of it is 0
+                L += v.y * ex2(v.x - M);
             }
-            uint4* dst = reinterpret_cast<uint4*>(bt.ext + sd.ext_off + ((int64_t)s * R_pad + row) * kExtCols);
-            dst[0] = make_uint4(w0, w1, 0u, 0u);
-            dst[1] = make_uint4(0u, 0u, 0u, 0u);
         }
+    }
+    part[j][threadIdx.x & (kCombRows - 1)] = make_float2(M, L);
+    __syncthreads();
+    if (j != 0 || row >= rows) return;
+    float off = 0.f;
+    if (row < R) {
+        float Mx = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) Mx = fmaxf(Mx, part[k][threadIdx.x].x);
+        float Lx = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 v = part[k][threadIdx.x];
+            if (v.x != -INFINITY) Lx += v.y * ex2(v.x - Mx);
+        }
+        off = Mx + log2f(Lx) + log2f((float)G);
+        bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
+    }
+    if (bt.ext) {
+        // the tcgen05 pass 2 adds -off / scale_log2e to the logit inside the contraction
+        // (one more K-step against a column of ones): three bf16 terms carry it to ~24 bits
+        uint32_t w0 = 0, w1 = 0;
+        if (row < R) {
+            const float x = -off / bt.scale_log2e;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+            const float r1 = x - __bfloat162float(hi);
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+            w0 = (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(mid) << 16);
+            w1 = (uint32_t)__bfloat16_as_ushort(lo);
+        } else {
+            w0 = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(-1e30f));   // exp2 of it is 0
+        }
+        uint4* dst = reinterpret_cast<uint4*>(bt.ext + sd.ext_off + ((int64_t)s * rows + row) * kExtCols);
+        dst[0] = make_uint4(w0, w1, 0u, 0u);
+        dst[1] = make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
@@ -484,10 +519,21 @@ cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+int64_t combine_blocks(const ScoreBatch& b) {
+    const int G = b.n_q_heads / b.n_kv_heads;
+    const int64_t nS = (int64_t)b.n_layers * b.n_kv_heads;
+    int64_t nb = 0;
+    for (int i = 0; i < b.n; ++i) {
+        const int64_t R = (int64_t)b.s[i].m * G;
+        const int64_t rows = b.ext ? rows_pad128(R) : R;
+        nb += nS * ((rows + kCombRows - 1) / kCombRows);
+    }
+    return nb;
+}
+
 cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
     const int G = b.n_q_heads / b.n_kv_heads;
-    const int nS = b.n_layers * b.n_kv_heads;
-    k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
+    k_combine<<<(unsigned)combine_blocks(b), kThreads, 0, st>>>(b, G);
     return cudaGetLastError();
 }
 
@@ -520,7 +566,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     stage_mark(b.timer, kStageStart, st);
     k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
     stage_mark(b.timer, kStageStats, st);
-    k_combine<<<(unsigned)(b.n * nS), kThreads, 0, st>>>(b, G);
+    k_combine<<<(unsigned)combine_blocks(b), kThreads, 0, st>>>(b, G);
     stage_mark(b.timer, kStageCombine, st);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
     stage_mark(b.timer, kStageAccum, st);
@@ -534,7 +580,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
 cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_t* err,
                             cudaError_t (*combine)(const ScoreBatch&, cudaStream_t));
 
-cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
+cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms, int* path_out) {
     const int G = b_in.n_q_heads / b_in.n_kv_heads;
     // finalize block ranges follow this file's finalize tile
     ScoreBatch* bp = new ScoreBatch(b_in);
@@ -553,10 +599,11 @@ cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
             delete w;
             ScoreBatch* v = new ScoreBatch(b);
             v->use_tc = 0;
-            e = launch_score(*v, st, num_sms);
+            e = launch_score(*v, st, num_sms, path_out);
             delete v;
             return e;
         }
+        *path_out = 2;
         if (e == cudaSuccess) {
             launch_finalize(*w, st);
             stage_mark(w->timer, kStageFinalize, st);
@@ -565,6 +612,7 @@ cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms) {
         delete w;
         return e;
     }
+    *path_out = 1;
     if (b.head_dim == 128) {
         if (G == 4) return launch_dg<128, 4>(b, st);
         if (G == 2) return launch_dg<128, 2>(b, st);

@@ -29,6 +29,7 @@ def _run(name, keep, senders=None):
     f.run()
     c.sync_status()
     torch.cuda.synchronize()
+    assert c.score_path() == 2, "full-size workloads run the tcgen05 logit passes"
     return spec, w, f
 
 

@@ -60,6 +60,7 @@ def test_parity(case, kernel):
         pytest.skip("shape outside the tcgen05 score path")
     w = _workload(name, shape, Ts, m)
     f = run_path(w, keep, score_kernel=kernel, **extra)
+    assert f.cb.score_path() == kernel, "the requested logit-pass kernels did not run"
     kw = dict(p=extra.get("p", 2.0), alpha=extra.get("alpha", 2.0), pool_w=extra.get("pool_width", 7),
               span_w=extra.get("span_width", 16))
     for i, s in enumerate(w.senders):
