@@ -181,16 +181,23 @@ class ClockSampler:
                 "power_w_max": max(x[3] for x in window)}
 
 
+# the sources whose SHA-256 (concatenated in this order) an ncu summary records
+KERNEL_SOURCES = ("cb_score_tc.cu", "cb_sm100.cuh", "cb_internal.cuh")
+
+
 def traffic_for(kernel: str, workload: str):
     """DRAM bytes (read + write) per launch of `kernel` on `workload` from the committed ncu
     summary, or None when that summary was taken on a different build of the kernel source."""
     import hashlib
     import re
     path = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
-    src = os.path.join(ROOT, "paper_2609_32046_gb300", "csrc", "cb_score_tc.cu")
+    csrc = os.path.join(ROOT, "paper_2609_32046_gb300", "csrc")
     try:
         text = open(path).read()
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        h = hashlib.sha256()
+        for f in KERNEL_SOURCES:
+            h.update(open(os.path.join(csrc, f), "rb").read())
+        sha = h.hexdigest()
         m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
         m_tr = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
         if m_sha and m_tr and m_sha.group(1) == sha:
@@ -460,6 +467,7 @@ def run_ours(args):
             "note": "max(HBM time of the algorithmic bytes, tensor time of both QK^T passes) / step time",
         },
         "gpu_launches": launches_per_step * args.steps,
+        "score_kernels": {2: "tcgen05", 1: "mma.sync"}.get(c.score_path(), "none"),
         "clocks": sampler.summary(t_wall0, t_wall1),
     }
     if e2e:
