@@ -38,8 +38,7 @@ void stage_mark(StageTimer* t, int stage, cudaStream_t st) {
     }
     cudaEvent_t e = t->pool[t->used++];
     if (cudaEventRecord(e, st) != cudaSuccess) { cudaGetLastError(); return; }
-    t->marks.emplace_back(stage, e);
-    if (stage == kStageStart) ++t->calls;
+    t->marks.emplace_back(stage, e);   // one call may hold several sender batches: cb_score counts calls
 }
 }  // namespace cbk
 
@@ -341,6 +340,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         delete bt;
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "score launch failed: %s", cudaGetErrorString(e));
     }
+    if (ctx->timer) ++ctx->timer->calls;
     return CB_OK;
 }
 

@@ -36,6 +36,8 @@ CASES = [
     ("pool3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=3)),
     ("pool5_p3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=5, p=3.0)),
     ("tail_1_position", (1, 8, 2, 128), [123], 8, 0.5, {}),
+    # more senders than one tcgen05 launch takes (32): two launches per pass
+    ("forty_senders", (1, 8, 2, 128), [97 + 13 * i for i in range(40)], 8, 0.3, {}),
 ]
 
 
@@ -190,3 +192,23 @@ def test_error_paths():
     c.sync_status()                             # the error word was cleared
     assert torch.equal(ko[:, :, 4], K[:, :, 7])
     assert not ko[:, :, 5].any()
+
+
+def test_stage_timing_counts_calls_across_sender_batches():
+    """Stage timing covers every sender batch of a call and counts cb_score calls, not batches."""
+    name, shape, Ts, m, keep, extra = [c for c in CASES if c[0] == "forty_senders"][0]
+    w = _workload(name, shape, Ts, m)
+    c = make_cb(w.spec.shape, max(Ts), m, len(Ts), score_kernel=2)
+    Ks = [s.K.cuda() for s in w.senders]
+    Qs = [w.queries[s.task].cuda() for s in w.senders]
+    S = [torch.empty(s.T, device="cuda") for s in w.senders]
+    c.enable_stage_timing(True)
+    c.stage_times()
+    for _ in range(3):
+        c.score(Ks, Qs, S)
+    st, calls = c.stage_times()
+    c.sync_status()
+    assert c.score_path() == 2
+    assert calls == 3
+    assert all(v > 0 for v in st.values()), st
+
