@@ -330,9 +330,13 @@ def run_ours(args):
                      spec.m, max(spec.T), len(senders))
     f = cb.Filter(c, senders, queries, keep, device=dev)
     stream = torch.cuda.current_stream(dev)
+    n_send = len(senders)
+    # --wave w: senders in waves on two streams (a wave's selection and compaction queued beside the
+    # next wave's scoring); sequential by default, which measured the same or faster on GB300
+    wave = args.wave if args.wave else 0
 
     for _ in range(args.warmup):
-        f.run(stream)
+        f.run(stream, wave=wave)
     c.sync_status(stream)
 
     c.enable_stage_timing(True)
@@ -348,6 +352,9 @@ def run_ours(args):
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for k in range(args.steps):
+        if wave:
+            f.run(stream, wave=wave)             # selection + compaction overlap the next wave's scoring
+            continue
         ev[4 * k].record(stream)
         f.score(stream)
         ev[4 * k + 1].record(stream)
@@ -366,18 +373,36 @@ def run_ours(args):
     stage_avg = {k: v / max(1, stage_calls) for k, v in stage_ms.items()}
     ms = start.elapsed_time(end)
     ms_max = max_over_ranks(ws, ms)
+    n_split = args.steps
+    if wave:
+        # per-step split of the three calls, from a few sequential steps after the timed region
+        n_split = min(args.steps, 3)
+        for k in range(n_split):
+            ev[4 * k].record(stream)
+            f.score(stream)
+            ev[4 * k + 1].record(stream)
+            f.select(stream)
+            ev[4 * k + 2].record(stream)
+            f.compact(stream)
+            ev[4 * k + 3].record(stream)
+        torch.cuda.synchronize(dev)
     per = {"score": [], "select": [], "compact": []}
-    for k in range(args.steps):
+    for k in range(n_split):
         per["score"].append(ev[4 * k].elapsed_time(ev[4 * k + 1]))
         per["select"].append(ev[4 * k + 1].elapsed_time(ev[4 * k + 2]))
         per["compact"].append(ev[4 * k + 2].elapsed_time(ev[4 * k + 3]))
     avg = {k: sum(v) / len(v) for k, v in per.items()}
 
     tokens_per_rank = sum(f.Ts)
-    n_send = len(senders)
-    score_batches = math.ceil(n_send / 64)
-    tc_batches = sum(math.ceil(min(64, n_send - 64 * b) / 32) for b in range(score_batches))
-    launches_per_step = (3 * tc_batches + score_batches) + 2 * score_batches   # score kernels, select, compact
+    def launches(n):
+        # per call group of <= 64 senders: statistics, combine and accumulation per <= 32 senders,
+        # then the two finalize kernels; one select and one compact launch per <= 64 senders
+        sb = math.ceil(n / 64)
+        tc = sum(math.ceil(min(64, n - 64 * b) / 32) for b in range(sb))
+        return 3 * tc + 2 * sb + sb + sb
+
+    waves = [min(wave, n_send - a) for a in range(0, n_send, wave)] if wave else [n_send]
+    launches_per_step = sum(launches(n) for n in waves)
     value = tokens_per_rank * ws * args.steps / (ms_max / 1e3)
     hbm_peak, tc_peak, tc_sus, src = peaks()
     tot_b, score_b, compact_b, flops = workload_bytes_flops(spec, keep)
@@ -403,7 +428,7 @@ def run_ours(args):
                 V.copy_(hv, non_blocking=True)
             for q, hq in zip(w.queries, hQ):
                 q.copy_(hq, non_blocking=True)
-            f.run(stream)
+            f.run(stream, wave=wave)
             hko.copy_(f.k_out, non_blocking=True)
             hvo.copy_(f.v_out, non_blocking=True)
             for x, hx in zip(f.idx, hidx):
@@ -436,7 +461,8 @@ def run_ours(args):
                    "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": keep,
                    "l2": "inputs larger than L2 (K+V %.2f GB per rank), no flush" % (
                        sum(K.numel() * 4 for K, _ in senders) / 1e9),
-                   "parallelism": "replicas" if ws > 1 else "single"},
+                   "parallelism": "replicas" if ws > 1 else "single",
+                   "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential"},
         "hbm_gbs": tot_b / step_s / 1e9,
         "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
         "algorithmic_bytes_per_step": tot_b,
@@ -495,6 +521,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-layers", type=int, default=4)
+    ap.add_argument("--wave", type=int, default=None,
+                    help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

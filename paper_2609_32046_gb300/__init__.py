@@ -62,11 +62,40 @@ class Filter:
     def compact(self, stream=None):
         self.cb.compact(self.Ks, self.Vs, self.idx, self.budgets, self.k_out, self.v_out, self.offsets, stream)
 
-    def run(self, stream=None):
-        self.score(stream)
-        self.select(stream)
-        self.compact(stream)
+    def run(self, stream=None, wave: Optional[int] = None):
+        """The whole path.  wave = None: score, select and compact every sender in turn on
+        `stream`.  wave = w: senders go in waves of w; a wave's selection and compaction run on a
+        second stream while the next wave is scored (compaction is bound by HBM bandwidth, the
+        scoring by the tensor pipe and exp2 throughput), and `stream` waits for both at the end.
+        Results are identical either way."""
+        n = len(self.Ks)
+        if not wave or wave >= n:
+            self.score(stream)
+            self.select(stream)
+            self.compact(stream)
+            return self
+        import torch
+        main = stream if stream is not None else torch.cuda.current_stream(self.Ks[0].device)
+        side = self._side_stream(main.device)
+        side.wait_stream(main)                       # inputs written on the caller's stream
+        for a in range(0, n, wave):
+            b = min(n, a + wave)
+            sl = slice(a, b)
+            self.cb.score(self.Ks[sl], self.Qs[sl], self.scores[sl], main)
+            done = torch.cuda.Event()
+            done.record(main)
+            side.wait_event(done)
+            self.cb.select(self.scores[sl], self.Ts[sl], self.budgets[sl], self.idx[sl], side)
+            self.cb.compact(self.Ks[sl], self.Vs[sl], self.idx[sl], self.budgets[sl], self.k_out, self.v_out,
+                            self.offsets[sl], side)
+        main.wait_stream(side)
         return self
+
+    def _side_stream(self, device):
+        import torch
+        if getattr(self, "_side", None) is None:
+            self._side = torch.cuda.Stream(device=device)
+        return self._side
 
     def indices(self) -> List:
         return [x[:b] for x, b in zip(self.idx, self.budgets)]

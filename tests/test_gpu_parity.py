@@ -212,3 +212,22 @@ def test_stage_timing_counts_calls_across_sender_batches():
     assert calls == 3
     assert all(v > 0 for v in st.values()), st
 
+
+def test_wave_schedule_matches_sequential():
+    """Selection and compaction on a second stream under the next wave's scoring: same bytes."""
+    name, shape, Ts, m, keep, extra = [c for c in CASES if c[0] == "forty_senders"][0]
+    w = _workload(name, shape, Ts, m)
+    c = make_cb(w.spec.shape, max(Ts), m, len(Ts), score_kernel=2)
+    pairs = [(s.K.cuda(), s.V.cuda()) for s in w.senders]
+    qs = [w.queries[s.task].cuda() for s in w.senders]
+    ref = cb.Filter(c, pairs, qs, keep).run()
+    got = cb.Filter(c, pairs, qs, keep).run(wave=7)
+    c.sync_status()
+    torch.cuda.synchronize()
+    for a, b in zip(ref.scores, got.scores):
+        assert torch.equal(a, b)
+    for a, b, B in zip(ref.idx, got.idx, ref.budgets):
+        assert torch.equal(a[:B], b[:B])
+    assert torch.equal(ref.k_out.view(torch.int16), got.k_out.view(torch.int16))
+    assert torch.equal(ref.v_out.view(torch.int16), got.v_out.view(torch.int16))
+
