@@ -52,10 +52,18 @@ def score(Kbits, Qbits, p=2.0, alpha=2.0, pool_w=7, scale=None) -> dict:
     Qt = pool(U, pool_w)
     # KV-group means b[l][g][r][t]
     b = a.reshape(nL, Hkv, G, m, T).mean(axis=2)
-    num = (pool(b, pool_w) ** p).mean(axis=2).sum(axis=(0, 1))
-    den = (pool(b.mean(axis=2), pool_w) ** p).sum(axis=(0, 1))
+    if math.isinf(p):
+        # the p -> infinity limit (App. D.2): largest pooled token attention over the largest
+        # pooled token mean, over all groups
+        num = pool(b, pool_w).max(axis=(0, 1, 2))
+        den = pool(b.mean(axis=2), pool_w).max(axis=(0, 1))
+        expo = 1.0
+    else:
+        num = (pool(b, pool_w) ** p).mean(axis=2).sum(axis=(0, 1))
+        den = (pool(b.mean(axis=2), pool_w) ** p).sum(axis=(0, 1))
+        expo = 1.0 / (p - 1.0)
     with np.errstate(divide="ignore", invalid="ignore"):
-        C = np.where(den > 0, (num / np.where(den > 0, den, 1.0)) ** (1.0 / (p - 1.0)), 1.0)
+        C = np.where(den > 0, (num / np.where(den > 0, den, 1.0)) ** expo, 1.0)
     S = Qt * C ** alpha
     return {"S": S, "Q": Qt, "C": C, "U": U, "N": num, "D": den, "a": a, "b": b}
 

@@ -159,7 +159,11 @@ int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, doub
  *   C_p,t = ( sum_s mean_r[Pool(b_{s,r,.})_t^p] / sum_s Pool(mean_r b_{s,r,.})_t^p )^(1/(p-1))
  *   S_t   = Q_t * C_p,t^alpha                                                     (CacheBack: p = alpha = 2)
  *
- * with C = 1 where the denominator is zero.  Outputs (any may be NULL), each [T]:
+ * with C = 1 where the denominator is zero.  p = +infinity takes the limit (App. D.2, parameter
+ * sensitivity: the largest pooled query-token attention against the largest pooled mean):
+ *   C_inf,t = max_{s,r} Pool(b_{s,r,.})_t / max_s Pool(mean_r b_{s,r,.})_t
+ * (the 1/m factor and the sums over s become 1 and maxima in the limit of the 1/(p-1) power);
+ * then N and D hold those maxima.  Outputs (any may be NULL), each [T]:
  *   S, Qt, C, U (the layer sum inside Pool, before pooling), N and D (numerator
  *   and denominator sums of C).
  * The work is split over the groups s = (l, g); each group's contributions are
@@ -172,6 +176,7 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
     if (st) return st;
     if (!K || !Q) return CBO_EINVAL;
     if (!(p > 1.0) || alpha < 0.0 || pool_w < 1 || (pool_w % 2) == 0) return CBO_EINVAL;
+    const int p_inf = isinf(p);
     const int64_t T = dm->T;
     const int m = dm->m, Hq = dm->n_q_heads, Hkv = dm->n_kv_heads, G = Hq / Hkv;
     const int nS = dm->n_layers * Hkv;
@@ -211,7 +216,10 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
             for (int r = 0; r < m; ++r) {
                 const double *br = b + (int64_t)r * T;
                 cbo_pool(br, pooled, T, pool_w);
-                for (int64_t t = 0; t < T; ++t) Ns[t] += pow(pooled[t], p) / m;
+                if (p_inf)
+                    for (int64_t t = 0; t < T; ++t) Ns[t] = pooled[t] > Ns[t] ? pooled[t] : Ns[t];
+                else
+                    for (int64_t t = 0; t < T; ++t) Ns[t] += pow(pooled[t], p) / m;
             }
             /* denominator: Pool(mean over r of b_{s,r,.})^p */
             for (int r = 0; r < m; ++r) {
@@ -219,7 +227,7 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
                 for (int64_t t = 0; t < T; ++t) bbar[t] += br[t] / m;
             }
             cbo_pool(bbar, pooled, T, pool_w);
-            for (int64_t t = 0; t < T; ++t) Ds[t] = pow(pooled[t], p);
+            for (int64_t t = 0; t < T; ++t) Ds[t] = p_inf ? pooled[t] : pow(pooled[t], p);
         }
         free(kt); free(b); free(z); free(a); free(pooled); free(bbar);
     }
@@ -235,13 +243,19 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
     }
     for (int s = 0; s < nS; ++s)
         for (int64_t t = 0; t < T; ++t) {
+            const double n_s = part[((int64_t)s * 3 + 1) * T + t], d_s = part[((int64_t)s * 3 + 2) * T + t];
             Usum[t] += part[((int64_t)s * 3 + 0) * T + t];
-            Nsum[t] += part[((int64_t)s * 3 + 1) * T + t];
-            Dsum[t] += part[((int64_t)s * 3 + 2) * T + t];
+            if (p_inf) {   /* maxima over the groups; every partial is >= 0 and the sums start at 0 */
+                Nsum[t] = n_s > Nsum[t] ? n_s : Nsum[t];
+                Dsum[t] = d_s > Dsum[t] ? d_s : Dsum[t];
+            } else {
+                Nsum[t] += n_s;
+                Dsum[t] += d_s;
+            }
         }
     cbo_pool(Usum, Qv, T, pool_w);
     for (int64_t t = 0; t < T; ++t) {
-        double c = Dsum[t] > 0.0 ? pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0)) : 1.0;
+        double c = Dsum[t] > 0.0 ? (p_inf ? Nsum[t] / Dsum[t] : pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))) : 1.0;
         if (S) S[t] = Qv[t] * pow(c, alpha);
         if (Qt) Qt[t] = Qv[t];
         if (C) C[t] = c;

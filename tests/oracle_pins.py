@@ -240,6 +240,45 @@ def pin_brute(o):
             assert o.select(r["S"], B).tolist() == brute.select(r["S"], B).tolist()
 
 
+def pin_p_infinity(o):
+    """p = infinity (App. D.2): C = max_{s,r} Pool(b) / max_s Pool(mean_r b), pinned by
+    (i) the literal numpy restatement, (ii) the limit of the finite-p oracle, which for any p
+    lies within factors (A/B)^(1/(p-1)) (m nS)^(-1/(p-1)) and (A/B)^(1/(p-1)) nS^(1/(p-1)) of
+    C_inf (A, B the two maxima), (iii) one group without pooling, where C = max_r b / mean_r b
+    with b from torch's SDPA, and (iv) one query token, where C = 1."""
+    inf = float("inf")
+    for (nL, Hq, Hkv, d, T, m, w) in ((2, 4, 2, 32, 61, 5, 7), (1, 8, 2, 16, 40, 3, 3)):
+        K, _, Q = _rand_case(nL, Hq, Hkv, d, T, m, seed=T + 7 * m)
+        r = o.score(K, Q, p=inf, alpha=2.0, pool_w=w)
+        b = brute.score(_bits(K), _bits(Q), p=inf, alpha=2.0, pool_w=w)
+        for k in ("S", "C", "N", "D"):
+            assert _rel(r[k], b[k]) < 1e-12, (k, _rel(r[k], b[k]))
+    # (ii) the finite-p limit, on a case small enough that b^p stays far from underflow
+    nL, Hq, Hkv, d, T, m = 2, 4, 2, 16, 24, 4
+    K, _, Q = _rand_case(nL, Hq, Hkv, d, T, m, seed=77)
+    ri = o.score(K, Q, p=inf, alpha=1.0)
+    A, B = ri["N"], ri["D"]
+    nS = nL * Hkv
+    for p in (24.0, 48.0):
+        rp = o.score(K, Q, p=p, alpha=1.0)
+        e = 1.0 / (p - 1.0)
+        ratio = rp["C"] / ri["C"]
+        lo = (A / B) ** e * (m * nS) ** (-e)
+        hi = (A / B) ** e * nS ** e
+        assert np.all(ratio >= lo * (1 - 1e-12)) and np.all(ratio <= hi * (1 + 1e-12)), p
+    # (iii) one group, no pooling
+    K1, _, Q1 = _rand_case(1, 2, 1, 16, 30, 4, seed=5)
+    r1 = o.score(K1, Q1, p=inf, alpha=1.0, pool_w=1)
+    Qd = Q1.to(torch.float64).permute(0, 2, 1, 3)                     # [1][Hq][m][d]
+    Kd = K1.to(torch.float64).expand(1, 2, 30, 16)
+    eye = torch.eye(30, dtype=torch.float64).expand(1, 2, 30, 30)
+    a = torch.nn.functional.scaled_dot_product_attention(Qd, Kd, eye, scale=0.25).numpy()   # [1][2][4][30]
+    bb = a[0].mean(axis=0)                                              # [m][T]: mean over the group's heads
+    assert _rel(r1["C"], bb.max(axis=0) / bb.mean(axis=0)) < 1e-12
+    # (iv) one query token
+    assert np.allclose(o.score(K, Q[:, :1].contiguous(), p=inf)["C"], 1.0, rtol=1e-13, atol=0)
+
+
 # --------------------------------------------------------------------------
 # selection (App. C.2)
 # --------------------------------------------------------------------------
@@ -305,6 +344,6 @@ def pin_compact(o):
 ALL_PINS = [
     pin_pool_one_hot, pin_pool_library, pin_attention_sdpa, pin_one_hot_closed_form,
     pin_zero_denominator, pin_variance_identity, pin_identical_keys, pin_invariants,
-    pin_special_cases, pin_equivariance, pin_brute, pin_select_golden, pin_select_integrity,
+    pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_select_golden, pin_select_integrity,
     pin_compact,
 ]

@@ -29,13 +29,18 @@ MUTANTS = [
     ("numerator_unpooled", "cbo_pool(br, pooled, T, pool_w);", "cbo_pool(br, pooled, T, 1);"),
     ("denominator_unpooled", "cbo_pool(bbar, pooled, T, pool_w);", "cbo_pool(bbar, pooled, T, 1);"),
     ("numerator_power_fixed_2", "Ns[t] += pow(pooled[t], p) / m;", "Ns[t] += pooled[t] * pooled[t] / m;"),
-    ("denominator_power_dropped", "Ds[t] = pow(pooled[t], p);", "Ds[t] = pooled[t];"),
+    ("denominator_power_dropped", "Ds[t] = p_inf ? pooled[t] : pow(pooled[t], p);", "Ds[t] = pooled[t];"),
     ("numerator_sum_not_mean", "Ns[t] += pow(pooled[t], p) / m;", "Ns[t] += pow(pooled[t], p);"),
     ("mean_query_attention_unpooled", "cbo_pool(Usum, Qv, T, pool_w);", "cbo_pool(Usum, Qv, T, 1);"),
     ("correction_exponent", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))", "pow(Nsum[t] / Dsum[t], 1.0 / p)"),
     ("correction_ratio_inverted", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))", "pow(Dsum[t] / Nsum[t], 1.0 / (p - 1.0))"),
     ("strength_exponent_dropped", "if (S) S[t] = Qv[t] * pow(c, alpha);", "if (S) S[t] = Qv[t] * c;"),
-    ("zero_denominator_gives_0", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0)) : 1.0;", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0)) : 0.0;"),
+    ("zero_denominator_gives_0", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))) : 1.0;", "pow(Nsum[t] / Dsum[t], 1.0 / (p - 1.0))) : 0.0;"),
+    ("p_inf_groups_summed", "Nsum[t] = n_s > Nsum[t] ? n_s : Nsum[t];", "Nsum[t] += n_s;"),
+    ("p_inf_denominator_groups_summed", "Dsum[t] = d_s > Dsum[t] ? d_s : Dsum[t];", "Dsum[t] += d_s;"),
+    ("p_inf_tokens_averaged", "Ns[t] = pooled[t] > Ns[t] ? pooled[t] : Ns[t];", "Ns[t] += pooled[t] / m;"),
+    ("p_inf_denominator_squared", "Ds[t] = p_inf ? pooled[t] : pow(pooled[t], p);", "Ds[t] = p_inf ? pooled[t] * pooled[t] : pow(pooled[t], p);"),
+    ("p_inf_ratio_inverted", "(p_inf ? Nsum[t] / Dsum[t] :", "(p_inf ? Dsum[t] / Nsum[t] :"),
     ("pool_window_too_wide", "int64_t half = w / 2;", "int64_t half = w / 2 + 1;"),
     ("pool_window_shifted", "int64_t hi = t + half > T - 1 ? T - 1 : t + half;", "int64_t hi = t + half + 1 > T - 1 ? T - 1 : t + half + 1;"),
     ("pool_min_not_max", "if (x[u] > mx) mx = x[u];", "if (x[u] < mx) mx = x[u];"),
