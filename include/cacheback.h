@@ -64,7 +64,9 @@ typedef struct cb_ctx cb_ctx; /* opaque; owns device scratch only */
  *   max_positions      upper bound on any sender's T (scratch is sized from it)
  *   max_senders        upper bound on senders per call
  *   softmax_scale      logit scale; 0 selects 1/sqrt(d)
- *   p, alpha           correction power p > 1 and strength alpha >= 0 (App. D.2)
+ *   p, alpha           correction power p > 1 and strength alpha >= 0 (App. D.2); p = +INFINITY
+ *                      takes the limit the parameter-sensitivity study names: C_t = largest pooled
+ *                      per-token attention / largest pooled token mean over the groups
  *   pool_width         Pool window, odd, 1..15 (7 in the paper; 1 disables pooling)
  *   span_width         span width for selection, 1..256 (16 in the paper; 1 ranks positions)
  *   n_sink, n_latent   forced positions: the first n_sink and the last n_latent (1 and 40)

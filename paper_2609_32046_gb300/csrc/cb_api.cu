@@ -183,7 +183,8 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
         return fail(nullptr, CB_ESHAPE, "max_positions must be in [1, 2^31)");
     if (c.max_senders < 1 || c.max_senders > 4096)
         return fail(nullptr, CB_ESHAPE, "max_senders %d not in [1, 4096]", c.max_senders);
-    if (!(std::isfinite(c.p) && c.p > 1.f)) return fail(nullptr, CB_EINVAL, "p must be finite and > 1");
+    if (!((std::isfinite(c.p) && c.p > 1.f) || (std::isinf(c.p) && c.p > 0.f)))
+        return fail(nullptr, CB_EINVAL, "p must be > 1 (or +infinity)");
     if (!(std::isfinite(c.alpha) && c.alpha >= 0.f)) return fail(nullptr, CB_EINVAL, "alpha must be finite and >= 0");
     if (!(std::isfinite(c.softmax_scale) && c.softmax_scale >= 0.f))
         return fail(nullptr, CB_EINVAL, "softmax_scale must be finite and >= 0");
@@ -300,6 +301,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->head_dim = c.head_dim;
         bt->scale_log2e = ctx->scale * 1.4426950408889634f;
         bt->p = c.p;
+        bt->p_inf = std::isinf(c.p) ? 1 : 0;
         bt->alpha = c.alpha;
         bt->pool_half = c.pool_width / 2;
         bt->use_tc = ctx->use_tc ? 1 : 0;

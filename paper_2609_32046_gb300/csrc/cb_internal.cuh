@@ -60,6 +60,7 @@ struct ScoreBatch {
     int32_t n_layers, n_q_heads, n_kv_heads, head_dim;
     float scale_log2e;        // softmax_scale * log2(e)
     float p, alpha;
+    int32_t p_inf;            // p = +infinity: N and D are maxima, C = N / D (App. D.2)
     int32_t pool_half;        // pool_width / 2
     int32_t use_tc;           // 1: tcgen05 passes, 0: mma.sync passes
     uint32_t* err;            // device error word

@@ -413,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
                 const float* row = bsm + rl * kBStride + col;
                 float mx = row[-ph];
                 for (int u = -ph + 1; u <= ph; ++u) mx = fmaxf(mx, row[u]);
-                nacc += powp(mx, bt.p, p2);
+                nacc = bt.p_inf ? fmaxf(nacc, mx) : nacc + powp(mx, bt.p, p2);
             }
             for (int k = threadIdx.x; k < kAccumPos; k += kThreads) {
                 float acc = 0.f;
@@ -432,8 +432,10 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
             const float inv_m = 1.f / (float)sd.m;
             float mx = bsum[col - ph];
             for (int u = -ph + 1; u <= ph; ++u) mx = fmaxf(mx, bsum[col + u]);
-            const float Nv = (nred[threadIdx.x] + nred[kAccumChunk + threadIdx.x]) * inv_m;
-            const float Dv = powp(mx * inv_m, bt.p, p2);
+            // p = infinity: the largest pooled token value and the pooled token mean itself
+            const float Nv = bt.p_inf ? fmaxf(nred[threadIdx.x], nred[kAccumChunk + threadIdx.x])
+                                      : (nred[threadIdx.x] + nred[kAccumChunk + threadIdx.x]) * inv_m;
+            const float Dv = bt.p_inf ? mx * inv_m : powp(mx * inv_m, bt.p, p2);
             const float Uv = bsum[col] * inv_m / (float)bt.n_kv_heads;
             float* part = bt.part + sd.part_off;
             part[((int64_t)0 * nS + s) * T + t] = Uv;
@@ -455,12 +457,21 @@ __global__ void __launch_bounds__(256) k_fin_sum(const __grid_constant__ ScoreBa
     const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
     if (t >= T) return;
     const float* part = bt.part + sd.part_off + t;
-    float U = 0.f, Nv = 0.f, Dv = 0.f;
+    float U = 0.f, Nv = 0.f, Dv = 0.f;   // p = infinity: N and D are maxima over the groups (all >= 0)
+    if (bt.p_inf) {
 #pragma unroll 6
-    for (int s = sl; s < nS; s += kFinSlices) {
-        U += __ldcs(part + (int64_t)s * T);
-        Nv += __ldcs(part + ((int64_t)nS + s) * T);
-        Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
+        for (int s = sl; s < nS; s += kFinSlices) {
+            U += __ldcs(part + (int64_t)s * T);
+            Nv = fmaxf(Nv, __ldcs(part + ((int64_t)nS + s) * T));
+            Dv = fmaxf(Dv, __ldcs(part + ((int64_t)2 * nS + s) * T));
+        }
+    } else {
+#pragma unroll 6
+        for (int s = sl; s < nS; s += kFinSlices) {
+            U += __ldcs(part + (int64_t)s * T);
+            Nv += __ldcs(part + ((int64_t)nS + s) * T);
+            Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
+        }
     }
     float* fin = bt.fin + sd.fin_off + (int64_t)sl * 3 * T + t;
     fin[0] = U;
@@ -490,8 +501,9 @@ __global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ 
         if (centre) {
 #pragma unroll
             for (int k = 0; k < kFinSlices; ++k) {
-                Nv += fin[((int64_t)k * 3 + 1) * T];
-                Dv += fin[((int64_t)k * 3 + 2) * T];
+                const float n_k = fin[((int64_t)k * 3 + 1) * T], d_k = fin[((int64_t)k * 3 + 2) * T];
+                Nv = bt.p_inf ? fmaxf(Nv, n_k) : Nv + n_k;
+                Dv = bt.p_inf ? fmaxf(Dv, d_k) : Dv + d_k;
             }
         }
     }
@@ -501,7 +513,7 @@ __global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ 
         const int ph = bt.pool_half;
         float Q = us[lp - ph];
         for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[lp + u]);
-        const float C = Dv > FLT_MIN ? powf(Nv / Dv, 1.f / (bt.p - 1.f)) : 1.f;
+        const float C = Dv > FLT_MIN ? (bt.p_inf ? Nv / Dv : powf(Nv / Dv, 1.f / (bt.p - 1.f))) : 1.f;
         const float S = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
         sd.scores[t] = S;
     }

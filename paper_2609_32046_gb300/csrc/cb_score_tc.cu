@@ -75,7 +75,7 @@ struct TcBatch {
     int32_t nL, Hq, Hkv, G;
     int32_t stages, rpad_max;
     float sl2e, p;
-    int32_t p_is_2, ph;
+    int32_t p_is_2, p_inf, ph;
     int64_t units1, units2;
     uint32_t* err;
     TcSender s[kMaxTcSenders];
@@ -491,7 +491,7 @@ __device__ __forceinline__ float pow_p(float x, float p) {
 // column, b = sum over the G heads of each token, then Pool over positions and the sums.
 template <int G, int PH, bool P2>
 __device__ __forceinline__ void accum_block(const float (&v)[32], uint64_t cc, bool valid, bool all_valid, float p,
-                                            float (&nacc)[2], float (&bsum)[2]) {
+                                            bool p_inf, float (&nacc)[2], float (&bsum)[2]) {
     float e[32];
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
@@ -520,6 +520,7 @@ __device__ __forceinline__ void accum_block(const float (&v)[32], uint64_t cc, b
         const float pk = lane_pool<PH>(b[k]);
         bsum[k & 1] += b[k];
         if (P2) nacc[k & 1] = fmaf(pk, pk, nacc[k & 1]);
+        else if (p_inf) nacc[k & 1] = fmaxf(nacc[k & 1], pk);   // p = infinity: largest pooled value
         else nacc[k & 1] += pow_p<false>(pk, p);
     }
 }
@@ -729,6 +730,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                         const float pk = lane_pool<PH>(b[k]);
                         bsum2[k & 1] += b[k];
                         if (P2) nacc2[k & 1] = fmaf(pk, pk, nacc2[k & 1]);
+                        else if (bt.p_inf) nacc2[k & 1] = fmaxf(nacc2[k & 1], pk);
                         else nacc2[k & 1] += pow_p<false>(pk, bt.p);
                     }
                 } else {
@@ -738,7 +740,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                         float v[32];
                         tmem_ld32(ta + col, v);
                         tmem_wait_ld();
-                        accum_block<G, PH, P2>(v, cc, valid, all_valid, bt.p, nacc2, bsum2);
+                        accum_block<G, PH, P2>(v, cc, valid, all_valid, bt.p, bt.p_inf, nacc2, bsum2);
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -746,7 +748,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 }
             }
             if (!ok) break;
-            float nacc = nacc2[0] + nacc2[1], bsum = bsum2[0] + bsum2[1];
+            // p = infinity keeps the largest pooled token value instead of the sum of powers
+            const bool p_inf = !P2 && bt.p_inf;
+            float nacc = p_inf ? fmaxf(nacc2[0], nacc2[1]) : nacc2[0] + nacc2[1];
+            float bsum = bsum2[0] + bsum2[1];
             // the two column halves of the group add up their sums; half 0 writes the results
             const int tp = (int)(gt & 1);
             float2* xs = xch + ((tp * 2 + grp) * 4 + sp) * 32;
@@ -758,13 +763,13 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             } else {
                 if (!(ok = wait_bar(xb, (uint32_t)((gt >> 1) & 1), ctl, bt.err, 14))) break;
                 const float2 o = xs[lane];
-                nacc += o.x;
+                nacc = p_inf ? fmaxf(nacc, o.x) : nacc + o.x;
                 bsum += o.y;
                 const float pb = lane_pool<PH>(bsum * inv_m);
                 if (valid && lane >= kMargin && lane < kMargin + kOutW) {
                     part[pos] = bsum * inv_mh;
-                    part[nST + pos] = nacc * inv_m;
-                    part[2 * nST + pos] = pow_p<P2>(pb, bt.p);
+                    part[nST + pos] = p_inf ? nacc : nacc * inv_m;
+                    part[2 * nST + pos] = p_inf ? pb : pow_p<P2>(pb, bt.p);
                 }
             }
             ++gt;
@@ -869,6 +874,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         tb->sl2e = b.scale_log2e;
         tb->p = b.p;
         tb->p_is_2 = b.p == 2.f;
+        tb->p_inf = b.p_inf;
         tb->ph = b.pool_half;
         tb->err = err;
         int rpad_max = 128;

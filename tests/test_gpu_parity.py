@@ -36,6 +36,10 @@ CASES = [
     ("pool3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=3)),
     ("pool5_p3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=5, p=3.0)),
     ("tail_1_position", (1, 8, 2, 128), [123], 8, 0.5, {}),
+    # p = infinity (App. D.2): maxima instead of sums of powers
+    ("p_inf_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(p=float("inf"))),
+    ("p_inf_g2_pool5", (2, 8, 4, 128), [611], 20, 0.3, dict(p=float("inf"), pool_width=5, alpha=3.0)),
+    ("p_inf_d64", (2, 8, 2, 64), [600], 12, 0.2, dict(p=float("inf"))),
     # more senders than one tcgen05 launch takes (32): two launches per pass
     ("forty_senders", (1, 8, 2, 128), [97 + 13 * i for i in range(40)], 8, 0.3, {}),
 ]
