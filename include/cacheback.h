@@ -162,6 +162,27 @@ cb_status cb_compact(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t
                      const int64_t *budget, void *k_out, void *v_out, int64_t out_capacity,
                      const int64_t *out_offset, int64_t o_layer, int64_t o_head, void *stream);
 
+/*
+ * Message rows by index (Sec. 3.1 "State Representation", App. C.3 "Message encoding").  The
+ * continuous-row encoding sends one row of the sender's per-position table (its hidden states:
+ * 8 KiB per position for Qwen3-8B) for every selected position; the token-ID encoding sends the
+ * selected source positions as token IDs (a table of 4-byte rows) and the latent positions as
+ * continuous rows.  Both are this gather, for each sender i:
+ *     out row (out_offset[i] + j) = row idx[i][j] of src[i],   j < count[i]
+ *   src[i]       device table, row t (t < T[i]) at src[i] + t * src_stride bytes
+ *   row_bytes    bytes per row, a positive multiple of 4 (src_stride, out_stride likewise, >= row_bytes)
+ *   idx[i]       device int32 [count[i]] (e.g. cb_select's output or a sub-range of it)
+ *   out          device buffer, row r at out + r * out_stride bytes, r < out_capacity
+ * Pointers need 4-byte alignment; rows of 16-byte multiples at 16-byte aligned addresses move
+ * as 16-byte pieces.  Asynchronous on `stream`; the caller owns every buffer.  Host errors: CB_EINVAL (NULL pointers, bad sizes
+ * or strides, host memory), CB_ESHAPE (n < 1, T < 1), CB_EBUDGET (count < 0 or rows past
+ * out_capacity).  An index outside [0, T[i]) skips its row and is reported by cb_sync_status as
+ * CB_EDEVICE.
+ */
+cb_status cb_gather(cb_ctx *ctx, int32_t n, const void *const *src, const int64_t *T, int64_t src_stride,
+                    int64_t row_bytes, const int32_t *const *idx, const int64_t *count, void *out,
+                    int64_t out_capacity, const int64_t *out_offset, int64_t out_stride, void *stream);
+
 /* Wait for `stream`, then report (and clear) errors the kernels recorded on the device
  * (CB_EDEVICE) or a failed launch (CB_ECUDA).  Blocks the host. */
 cb_status cb_sync_status(cb_ctx *ctx, void *stream);

@@ -73,6 +73,9 @@ class Oracle:
         lib.cbo_compact.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_int64, _P, _P,
                                     ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
         lib.cbo_compact.restype = ctypes.c_int
+        lib.cbo_gather.argtypes = [_P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, _P, ctypes.c_int64, _P,
+                                   ctypes.c_int64, ctypes.c_int64]
+        lib.cbo_gather.restype = ctypes.c_int
         lib.cbo_pool.argtypes = [_P, _P, ctypes.c_int64, ctypes.c_int32]
         lib.cbo_pool.restype = None
         lib.cbo_max_threads.restype = ctypes.c_int
@@ -167,6 +170,33 @@ class Oracle:
         if st != OK:
             raise RuntimeError("cbo_compact failed with status %d" % st)
         return out_k, out_v
+
+
+    def gather(self, table, idx, out=None, offset: int = 0) -> np.ndarray:
+        """Message rows (App. C.3): out[offset + j] = table[idx[j]] as raw bytes.  table: numpy
+        array or tensor with one row per position (its leading axis)."""
+        tb = np.ascontiguousarray(self._raw(table))
+        T = tb.shape[0]
+        row_bytes = tb[0].nbytes if T else 0
+        idx = np.ascontiguousarray(idx, dtype=np.int32)
+        if out is None:
+            out = np.zeros((offset + idx.shape[0],) + tb.shape[1:], dtype=tb.dtype)
+        assert out.flags.c_contiguous and out.dtype == tb.dtype and out.shape[1:] == tb.shape[1:]
+        st = self.lib.cbo_gather(tb.ctypes.data, T, row_bytes, row_bytes, idx.ctypes.data, idx.shape[0],
+                                 out.ctypes.data, offset, row_bytes)
+        if st != OK:
+            raise RuntimeError("cbo_gather failed with status %d" % st)
+        return out
+
+    @staticmethod
+    def _raw(x) -> np.ndarray:
+        if isinstance(x, np.ndarray):
+            return x
+        import torch
+        x = x.detach().cpu().contiguous()
+        if x.dtype in (torch.bfloat16, torch.float16):
+            return x.view(torch.int16).numpy().view(np.uint16)
+        return x.numpy()
 
 
 def budget(T: int, keep: float) -> int:

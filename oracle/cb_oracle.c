@@ -415,4 +415,22 @@ int cbo_compact(const cbo_dims *dm, const uint16_t *K, const uint16_t *V, const 
     return CBO_OK;
 }
 
+/*
+ * Message rows (Sec. 3.1 "State Representation", App. C.3 "Message encoding"): the
+ * continuous-row encoding sends the sender's per-position row (hidden state) of every selected
+ * position, the token-ID encoding the token ID (a 4-byte row) of every selected source position:
+ *   out row (off + j) = src row idx[j],   j < count,
+ * rows of row_bytes raw bytes, row t of src at src + t * src_stride, row r of out at
+ * out + r * out_stride.
+ */
+int cbo_gather(const uint8_t *src, int64_t T, int64_t src_stride, int64_t row_bytes, const int32_t *idx,
+               int64_t count, uint8_t *out, int64_t off, int64_t out_stride) {
+    if (!src || !out || (count > 0 && !idx) || T < 1 || count < 0 || row_bytes < 1) return CBO_EINVAL;
+    for (int64_t j = 0; j < count; ++j)
+        if (idx[j] < 0 || idx[j] >= T) return CBO_EINVAL;
+    for (int64_t j = 0; j < count; ++j)
+        memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);
+    return CBO_OK;
+}
+
 int cbo_max_threads(void) { return omp_get_max_threads(); }

@@ -99,3 +99,34 @@ class Filter:
 
     def indices(self) -> List:
         return [x[:b] for x, b in zip(self.idx, self.budgets)]
+
+    # -- message encodings (Sec. 3.1 "State Representation", App. C.3) ------------------
+    def message_rows(self, tables: Sequence, stream=None):
+        """Continuous-row encoding: every selected position as one row of the sender's
+        per-position table (e.g. hidden states [T_i][hidden]); senders back to back."""
+        import torch
+        out = torch.empty((max(self.capacity, 1),) + tuple(tables[0].shape[1:]), dtype=tables[0].dtype,
+                          device=tables[0].device)
+        self.cb.gather(tables, self.idx, self.budgets, out, self.offsets, stream)
+        return out[:self.capacity]
+
+    def message_token_ids(self, token_ids: Sequence, tables: Sequence, stream=None):
+        """Token-ID encoding: the selected source positions as token IDs (int32 [T_i] tables), the
+        latent positions (the last n_latent, always selected) as continuous rows.  Returns
+        (ids [sum_i (B_i - L_i)], rows [sum_i L_i][...]) with L_i = min(T_i, n_latent)."""
+        import torch
+        lat = [min(T, self.cb.cfg.n_latent) for T in self.Ts]
+        n_src = [b - l for b, l in zip(self.budgets, lat)]
+        id_off, row_off = [], []
+        a = r = 0
+        for ns, nl in zip(n_src, lat):
+            id_off.append(a); row_off.append(r)
+            a += ns; r += nl
+        dev = tables[0].device
+        ids = torch.empty(max(a, 1), dtype=torch.int32, device=dev)
+        rows = torch.empty((max(r, 1),) + tuple(tables[0].shape[1:]), dtype=tables[0].dtype, device=dev)
+        tabs = [t.view(-1, 1) for t in token_ids]
+        self.cb.gather(tabs, [x[:max(ns, 1)] for x, ns in zip(self.idx, n_src)], n_src, ids.view(-1, 1), id_off,
+                       stream)
+        self.cb.gather(tables, [x[ns:] for x, ns in zip(self.idx, n_src)], lat, rows, row_off, stream)
+        return ids[:a], rows[:r]

@@ -21,6 +21,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
             "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
+            "cb_gather",
             "cb_enable_stage_timing", "cb_stage_times"]
 
 
@@ -77,6 +78,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_compact.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), P, P, P, P, ctypes.c_int64, P,
                                ctypes.c_int64, ctypes.c_int64, P]
     lib.cb_compact.restype = ctypes.c_int
+    lib.cb_gather.argtypes = [P, ctypes.c_int32, P, P, ctypes.c_int64, ctypes.c_int64, P, P, P, ctypes.c_int64, P,
+                              ctypes.c_int64, P]
+    lib.cb_gather.restype = ctypes.c_int
     lib.cb_sync_status.argtypes = [P, P]
     lib.cb_sync_status.restype = ctypes.c_int
     lib.cb_destroy.argtypes = [P]
@@ -219,6 +223,27 @@ class CacheBack:
         self._check(self.lib.cb_compact(self.h, n, kv, ip, Ba, k_out.data_ptr(), v_out.data_ptr(),
                                         k_out.shape[2], Oa, k_out.stride(0), k_out.stride(1),
                                         _stream_handle(stream)))
+
+    def gather(self, tables: Sequence, idx: Sequence, counts: Sequence[int], out, offsets: Sequence[int],
+               stream=None):
+        """Message rows (App. C.3): out row offsets[i] + j = tables[i][idx[i][j]], j < counts[i].
+        tables: per-sender [T_i][...] device tensors with one row per position (same row size and
+        row stride); out: [capacity][...] with the same row size; idx: int32 device tensors."""
+        n = len(tables)
+        row_bytes = tables[0][0].numel() * tables[0].element_size()
+        src_stride = tables[0].stride(0) * tables[0].element_size()
+        for t in tables:
+            assert t[0].is_contiguous() and t.stride(0) * t.element_size() == src_stride
+            assert t[0].numel() * t.element_size() == row_bytes
+        assert out[0].numel() * out.element_size() == row_bytes and out[0].is_contiguous()
+        sp = _ptr_array([t.data_ptr() for t in tables])
+        Ta = _ptr_array([int(t.shape[0]) for t in tables], ctypes.c_int64)
+        ip = _ptr_array([x.data_ptr() for x in idx])
+        Ca = _ptr_array([int(c) for c in counts], ctypes.c_int64)
+        Oa = _ptr_array([int(o) for o in offsets], ctypes.c_int64)
+        self._check(self.lib.cb_gather(self.h, n, sp, Ta, src_stride, row_bytes, ip, Ca, out.data_ptr(),
+                                       out.shape[0], Oa, out.stride(0) * out.element_size(),
+                                       _stream_handle(stream)))
 
     STAGES = ("row_statistics", "statistics_combine", "normalised_accumulation", "finalize")
 

@@ -96,12 +96,12 @@ struct DeviceGuard {
     }
 };
 
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // The pointer must be device (or managed) memory on ctx's device.
-cb_status check_device_ptr(cb_ctx* ctx, const void* p, const char* what, int i) {
+cb_status check_device_ptr(cb_ctx* ctx, const void* p, const char* what, int i, int align = 16) {
     if (!p) return fail(ctx, CB_EINVAL, "%s[%d] is NULL", what, i);
-    if (!aligned16(p)) return fail(ctx, CB_EINVAL, "%s[%d] is not 16-byte aligned", what, i);
+    if (reinterpret_cast<uintptr_t>(p) % (uintptr_t)align != 0)
+        return fail(ctx, CB_EINVAL, "%s[%d] is not %d-byte aligned", what, i, align);
     cudaPointerAttributes a;
     cudaError_t e = cudaPointerGetAttributes(&a, p);
     if (e != cudaSuccess) {
@@ -497,6 +497,58 @@ cb_status cb_stage_times(cb_ctx* ctx, float* ms, int32_t* calls) {
     return CB_OK;
 }
 
+cb_status cb_gather(cb_ctx* ctx, int32_t n, const void* const* src, const int64_t* T, int64_t src_stride,
+                    int64_t row_bytes, const int32_t* const* idx, const int64_t* count, void* out,
+                    int64_t out_capacity, const int64_t* out_offset, int64_t out_stride, void* stream) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    if (n < 1) return fail(ctx, CB_ESHAPE, "n = %d < 1", n);
+    if (!src || !T || !idx || !count || !out_offset) return fail(ctx, CB_EINVAL, "src, T, idx, count or out_offset is NULL");
+    if (row_bytes <= 0 || row_bytes % 4 != 0) return fail(ctx, CB_EINVAL, "row_bytes %lld must be a positive multiple of 4",
+                                                          (long long)row_bytes);
+    if (src_stride < row_bytes || src_stride % 4 != 0 || out_stride < row_bytes || out_stride % 4 != 0)
+        return fail(ctx, CB_EINVAL, "strides must be multiples of 4 bytes and at least row_bytes");
+    if (out_capacity < 0) return fail(ctx, CB_EINVAL, "out_capacity < 0");
+    DeviceGuard dg(ctx->device);
+    if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
+    cb_status st;
+    if ((st = check_device_ptr(ctx, out, "out", 0, 4))) return st;
+    for (int i = 0; i < n; ++i) {
+        if (T[i] < 1) return fail(ctx, CB_ESHAPE, "T[%d] = %lld < 1", i, (long long)T[i]);
+        if (count[i] < 0) return fail(ctx, CB_EBUDGET, "count[%d] = %lld < 0", i, (long long)count[i]);
+        if (out_offset[i] < 0 || out_offset[i] + count[i] > out_capacity)
+            return fail(ctx, CB_EBUDGET, "sender %d: rows [%lld, %lld) exceed out_capacity %lld", i,
+                        (long long)out_offset[i], (long long)(out_offset[i] + count[i]), (long long)out_capacity);
+        if (count[i] * (row_bytes / 4) >= ((int64_t)1 << 40))
+            return fail(ctx, CB_ESHAPE, "sender %d: message too large", i);
+        if ((st = check_device_ptr(ctx, src[i], "src", i, 4))) return st;
+        if (count[i] > 0 && (st = check_device_ptr(ctx, idx[i], "idx", i, 4))) return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    for (int b0 = 0; b0 < n; b0 += cbk::kMaxBatch) {
+        const int nb = n - b0 < cbk::kMaxBatch ? n - b0 : cbk::kMaxBatch;
+        cbk::GatherBatch bt;
+        std::memset(&bt, 0, sizeof bt);
+        bt.n = nb;
+        bt.row_bytes = row_bytes;
+        bt.out = static_cast<uint8_t*>(out);
+        bt.out_stride = out_stride;
+        bt.err = ctx->err;
+        for (int k = 0; k < nb; ++k) {
+            cbk::GatherSender& d = bt.s[k];
+            d.src = static_cast<const uint8_t*>(src[b0 + k]);
+            d.idx = idx[b0 + k];
+            d.T = T[b0 + k];
+            d.src_stride = src_stride;
+            d.count = count[b0 + k];
+            d.out_off = out_offset[b0 + k];
+        }
+        cudaError_t e = cbk::launch_gather(bt, strm, ctx->num_sms);
+        if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "gather launch failed: %s", cudaGetErrorString(e));
+    }
+    return CB_OK;
+}
+
 cb_status cb_sync_status(cb_ctx* ctx, void* stream) {
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     DeviceGuard dg(ctx->device);
@@ -512,9 +564,10 @@ cb_status cb_sync_status(cb_ctx* ctx, void* stream) {
             return fail(ctx, CB_ETIMEOUT,
                         "a bounded device wait gave up (code 0x%x: bits 8+ name the wait); the results are invalid",
                         word);
-        return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s)", word,
+        return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s%s)", word,
                     (word & cbk::kErrCompactIndex) ? " compact index outside [0, T)" : "",
-                    (word & cbk::kErrSelectBudget) ? " select count mismatch" : "");
+                    (word & cbk::kErrSelectBudget) ? " select count mismatch" : "",
+                    (word & cbk::kErrGatherIndex) ? " gather index outside [0, T)" : "");
     }
     return CB_OK;
 }

@@ -28,6 +28,7 @@ constexpr int kMaxQueryTokens = 1024;
 constexpr uint32_t kErrCompactIndex = 1u;
 constexpr uint32_t kErrSelectBudget = 2u;
 constexpr uint32_t kErrTimeout = 4u;       // a bounded mbarrier wait gave up
+constexpr uint32_t kErrGatherIndex = 8u;   // a message-row index outside [0, T)
 
 // Optional per-kernel timing of the score step (owned by the context; see cb_stage_times).
 struct StageTimer;
@@ -117,6 +118,26 @@ struct CompactBatch {
     CompactSender s[kMaxBatch];
 };
 
+// Message rows (Sec. 3.1 "State Representation", App. C.3): row j of sender i's message is
+// row idx[j] of its per-position table.
+struct GatherSender {
+    const uint8_t* src;       // row t at src + t * src_stride (bytes)
+    const int32_t* idx;       // count indices into [0, T)
+    int64_t T;
+    int64_t src_stride;
+    int64_t count;
+    int64_t out_off;          // first output row of this sender
+};
+
+struct GatherBatch {
+    int32_t n;
+    int64_t row_bytes;        // bytes per row: a multiple of 4
+    uint8_t* out;             // row r at out + r * out_stride
+    int64_t out_stride;
+    uint32_t* err;
+    GatherSender s[kMaxBatch];
+};
+
 // Records the message cb_last_error(NULL) returns (entry points without a context).
 void set_context_free_error(const char* msg);
 
@@ -128,5 +149,6 @@ bool tc_path_supported(int head_dim, int G, int pool_half, int max_query_tokens)
 cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms, int* path_out);
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);
 cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms);
+cudaError_t launch_gather(const GatherBatch& b, cudaStream_t st, int num_sms);
 
 }  // namespace cbk

@@ -341,9 +341,20 @@ def pin_compact(o):
     assert not ko[:, :, :off].any() and not vo[:, :, :off].any()
 
 
+def pin_gather(o):
+    """Message rows (App. C.3) equal numpy fancy indexing, for hidden-state rows and token IDs."""
+    rng = np.random.default_rng(4)
+    rows = rng.integers(0, 1 << 16, size=(70, 48), dtype=np.uint16)
+    ids = rng.integers(0, 150000, size=70, dtype=np.int32)
+    idx = np.array([0, 3, 4, 17, 40, 41, 69], dtype=np.int32)
+    assert np.array_equal(o.gather(rows, idx, offset=2)[2:], rows[idx])
+    assert not o.gather(rows, idx, offset=2)[:2].any()
+    assert np.array_equal(o.gather(ids, idx), ids[idx])
+
+
 ALL_PINS = [
     pin_pool_one_hot, pin_pool_library, pin_attention_sdpa, pin_one_hot_closed_form,
     pin_zero_denominator, pin_variance_identity, pin_identical_keys, pin_invariants,
     pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_select_golden, pin_select_integrity,
-    pin_compact,
+    pin_compact, pin_gather,
 ]

@@ -54,6 +54,8 @@ MUTANTS = [
     ("short_span_mean_over_full_width_f32", "rank[j].mean = (double)(acc / (float)(hi - lo));", "rank[j].mean = (double)(acc / (float)span_w);"),
     ("ranking_ascending", "if (a->mean > b->mean) return -1;\n    if (a->mean < b->mean) return 1;", "if (a->mean < b->mean) return -1;\n    if (a->mean > b->mean) return 1;"),
     ("compact_offset_dropped", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + (off + j) * d;", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + j * d;"),
+    ("gather_offset_dropped", "memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);", "memcpy(out + j * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);"),
+    ("gather_row_shifted", "memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);", "memcpy(out + (off + j) * out_stride, src + (int64_t)(idx[j] + (idx[j] + 1 < T)) * src_stride, (size_t)row_bytes);"),
     ("compact_v_from_k", "memcpy(v_out + dst, V + src, sizeof(uint16_t) * (size_t)d);", "memcpy(v_out + dst, K + src, sizeof(uint16_t) * (size_t)d);"),
 ]
 
