@@ -132,6 +132,15 @@ cb_status cb_score(cb_ctx *ctx, int32_t n, const cb_kv *senders, const cb_query 
  * with keep = 1/r).  Pure host function; needs no context. */
 int64_t cb_budget(int64_t T, double keep);
 
+/* Budget of one hop of a sequential chain (App. C.2): the hop's cache holds T_old inherited
+ * positions (the previous message) followed by T_new new prompt and latent positions.
+ *   mode 0 (relative): B = T_old + ceil(keep * T_new)   (keep = 1/r, ceiling in double)
+ *   mode 1 (fixed):    B = min(B_max, T_old + T_new)
+ * clamped to [0, T_old + T_new].  Inherited and new positions are then ranked together by
+ * cb_select (only the first position and the last n_latent positions are forced).  Returns -1
+ * for negative sizes, an unknown mode or a negative B_max.  Pure host function. */
+int64_t cb_chain_budget(int64_t T_old, int64_t T_new, double keep, int32_t mode, int64_t B_max);
+
 /*
  * Select (App. C.2): for each sender i, write idx[i][0..budget[i]) (int32, device),
  * strictly ascending, containing the forced positions (the first n_sink and the last

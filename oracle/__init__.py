@@ -204,6 +204,19 @@ def budget(T: int, keep: float) -> int:
     return int(min(T, max(0, math.ceil(keep * T))))
 
 
+def chain_budget(T_old: int, T_new: int, keep: float = 0.0, mode: str = "relative", B_max: int = 0) -> int:
+    """One hop of a sequential chain (App. C.2): relative B = T_old + ceil(T_new / r) with r = 1/keep,
+    fixed B = min(B_max, T_old + T_new); at most T_old + T_new."""
+    T = T_old + T_new
+    if mode == "relative":
+        B = T_old + budget(T_new, keep)
+    elif mode == "fixed":
+        B = min(B_max, T)
+    else:
+        raise ValueError(mode)
+    return min(T, max(0, B))
+
+
 _DEFAULT: Optional[Oracle] = None
 
 

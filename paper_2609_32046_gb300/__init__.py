@@ -14,9 +14,9 @@ from __future__ import annotations
 from typing import List, Optional, Sequence
 
 from .binding import (CB_EBUDGET, CB_ECUDA, CB_EDEVICE, CB_EINVAL, CB_ENOMEM, CB_ESHAPE, CB_OK, EXPORTED,
-                      LIB_PATH, CacheBack, CBError, budget, load_library)
+                      LIB_PATH, CacheBack, CBError, budget, chain_budget, load_library)
 
-__all__ = ["CacheBack", "CBError", "budget", "load_library", "LIB_PATH", "EXPORTED", "Filter",
+__all__ = ["CacheBack", "CBError", "budget", "chain_budget", "load_library", "LIB_PATH", "EXPORTED", "Filter", "Chain",
            "CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_EDEVICE"]
 
 
@@ -130,3 +130,62 @@ class Filter:
                        stream)
         self.cb.gather(tables, [x[ns:] for x, ns in zip(self.idx, n_src)], lat, rows, row_off, stream)
         return ids[:a], rows[:r]
+
+
+class Chain:
+    """Sequential communication (App. C.2; the LongBench hops of Sec. 4): hop i's sender cache is
+    the previous hop's message (its selected K/V rows, in source order) followed by the hop's new
+    prompt and latent positions.  Each hop scores that whole cache against its receiver query,
+    selects B_i positions under the chain budget (inherited and new positions ranked together;
+    only the first and the current n_latent positions forced, so inherited latent positions may be
+    dropped) and compacts them into the front of the other of two cache buffers, which the next
+    hop extends.  Nothing is copied besides the compaction.
+
+    cb:        CacheBack sized for one sender with max_positions >= capacity
+    capacity:  the largest T_old + T_new of any hop
+    mode:      "relative" (B = T_old + ceil(keep T_new)) or "fixed" (B = min(B_max, T_old + T_new))
+    """
+
+    def __init__(self, cb: CacheBack, capacity: int, keep: float = 0.25, mode: str = "relative",
+                 B_max: int = 0, device=None):
+        import torch
+        self.cb, self.capacity, self.keep, self.mode, self.B_max = cb, int(capacity), keep, mode, B_max
+        c = cb.cfg
+        shape = (c.n_layers, c.n_kv_heads, self.capacity, c.head_dim)
+        self.K = [torch.empty(shape, dtype=torch.bfloat16, device=device) for _ in range(2)]
+        self.V = [torch.empty(shape, dtype=torch.bfloat16, device=device) for _ in range(2)]
+        self.cur = 0
+        self.T_old = 0
+
+    def new_slot(self, T_new: int):
+        """Views of the current buffer where the hop's T_new new positions go (after the message)."""
+        a, b = self.T_old, self.T_old + int(T_new)
+        if b > self.capacity:
+            raise ValueError("hop of %d positions exceeds the chain capacity %d" % (b, self.capacity))
+        return self.K[self.cur][:, :, a:b], self.V[self.cur][:, :, a:b]
+
+    def hop(self, Q, K_new=None, V_new=None, T_new: Optional[int] = None, stream=None) -> dict:
+        """One hop: K_new / V_new (or T_new positions already written through new_slot) join the
+        inherited message; returns the hop's cache views, scores, budget and selected indices."""
+        import torch
+        if K_new is not None:
+            T_new = int(K_new.shape[2])
+            k, v = self.new_slot(T_new)
+            k.copy_(K_new)
+            v.copy_(V_new)
+        T_old, T = self.T_old, self.T_old + int(T_new)
+        c = self.cb.cfg
+        B = chain_budget(T_old, T_new, self.keep, self.mode, self.B_max)
+        B = max(B, min(T, c.n_sink + c.n_latent))          # the forced positions always fit
+        Kv, Vv = self.K[self.cur][:, :, :T], self.V[self.cur][:, :, :T]
+        scores = torch.empty(T, dtype=torch.float32, device=Kv.device)
+        idx = torch.empty(max(B, 1), dtype=torch.int32, device=Kv.device)
+        self.cb.score([Kv], [Q], [scores], stream)
+        self.cb.select([scores], [T], [B], [idx], stream)
+        nxt = 1 - self.cur
+        self.cb.compact([Kv], [Vv], [idx], [B], self.K[nxt], self.V[nxt], [0], stream)
+        out = {"K": Kv, "V": Vv, "T_old": T_old, "T": T, "B": B, "scores": scores, "idx": idx[:B],
+               "message_K": self.K[nxt][:, :, :B], "message_V": self.V[nxt][:, :, :B]}
+        self.cur, self.T_old = nxt, B
+        return out
+

@@ -21,7 +21,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
             "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
-            "cb_gather",
+            "cb_gather", "cb_chain_budget",
             "cb_enable_stage_timing", "cb_stage_times"]
 
 
@@ -73,6 +73,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_score.restype = ctypes.c_int
     lib.cb_budget.argtypes = [ctypes.c_int64, ctypes.c_double]
     lib.cb_budget.restype = ctypes.c_int64
+    lib.cb_chain_budget.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.c_int32, ctypes.c_int64]
+    lib.cb_chain_budget.restype = ctypes.c_int64
     lib.cb_select.argtypes = [P, ctypes.c_int32, P, P, P, P, P]
     lib.cb_select.restype = ctypes.c_int
     lib.cb_compact.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), P, P, P, P, ctypes.c_int64, P,
@@ -105,6 +107,16 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
 def budget(T: int, keep: float) -> int:
     """ceil(keep * T) in double, clamped to [0, T] (App. C.2), computed by the library."""
     return int(load_library().cb_budget(int(T), float(keep)))
+
+
+def chain_budget(T_old: int, T_new: int, keep: float = 0.0, mode: str = "relative", B_max: int = 0) -> int:
+    """Budget of one hop of a sequential chain (App. C.2): relative T_old + ceil(keep T_new) or
+    fixed min(B_max, T_old + T_new), computed by the library."""
+    m = {"relative": 0, "fixed": 1}[mode]
+    b = int(load_library().cb_chain_budget(int(T_old), int(T_new), float(keep), m, int(B_max)))
+    if b < 0:
+        raise ValueError("invalid chain budget arguments")
+    return b
 
 
 def select_noalloc(scores: Sequence, Ts: Sequence[int], budgets: Sequence[int], idx: Sequence, n_sink: int = 1,

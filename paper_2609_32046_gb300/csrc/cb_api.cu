@@ -156,6 +156,16 @@ int64_t cb_budget(int64_t T, double keep) {
     return (int64_t)b;
 }
 
+int64_t cb_chain_budget(int64_t T_old, int64_t T_new, double keep, int32_t mode, int64_t B_max) {
+    if (T_old < 0 || T_new < 0) return -1;
+    const int64_t T = T_old + T_new;
+    int64_t B;
+    if (mode == 0) B = T_old + cb_budget(T_new, keep);
+    else if (mode == 1 && B_max >= 0) B = B_max < T ? B_max : T;
+    else return -1;
+    return B < 0 ? 0 : (B > T ? T : B);
+}
+
 const char* cb_last_error(const cb_ctx* ctx) { return ctx ? ctx->last_error.c_str() : g_create_error.c_str(); }
 
 int64_t cb_scratch_bytes(const cb_ctx* ctx) { return ctx ? ctx->scratch_bytes : 0; }

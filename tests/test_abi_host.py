@@ -56,6 +56,21 @@ def _cfg(lib, **kw):
     return c
 
 
+def test_chain_budget_matches_the_paper_rule(lib):
+    """App. C.2's two chain budgets, library against the oracle's restatement."""
+    import oracle
+    for T_old in (0, 1, 41, 2048, 6554):
+        for T_new in (0, 1, 40, 777, 25000, 61000):
+            for keep in (0.1, 0.25, 1 / 3, 0.5):
+                assert cb.chain_budget(T_old, T_new, keep) == oracle.chain_budget(T_old, T_new, keep)
+            for B_max in (0, 41, 4096, 10 ** 7):
+                assert cb.chain_budget(T_old, T_new, mode="fixed", B_max=B_max) == \
+                    oracle.chain_budget(T_old, T_new, mode="fixed", B_max=B_max)
+    assert cb.chain_budget(2048, 25000, 0.25) == 2048 + 6250          # inherited rows all count
+    assert lib.cb_chain_budget(-1, 5, 0.5, 0, 0) == -1 and lib.cb_chain_budget(5, 5, 0.5, 2, 0) == -1
+    assert lib.cb_chain_budget(5, 5, 0.5, 1, -1) == -1
+
+
 def test_defaults_follow_the_paper(lib):
     c = binding.cb_config()
     lib.cb_config_init(ctypes.byref(c))
