@@ -48,6 +48,7 @@ class _Dims(ctypes.Structure):
         ("head_dim", ctypes.c_int32), ("m", ctypes.c_int32), ("T", ctypes.c_int64),
         ("k_layer", ctypes.c_int64), ("k_head", ctypes.c_int64), ("k_pos", ctypes.c_int64),
         ("q_layer", ctypes.c_int64), ("q_tok", ctypes.c_int64), ("q_head", ctypes.c_int64),
+        ("s_layer", ctypes.c_int64), ("s_tok", ctypes.c_int64), ("s_head", ctypes.c_int64),
     ]
 
 
@@ -65,6 +66,11 @@ class Oracle:
         lib.cbo_score.restype = ctypes.c_int
         lib.cbo_attention.argtypes = [ctypes.POINTER(_Dims), _P, _P, ctypes.c_double, _P]
         lib.cbo_attention.restype = ctypes.c_int
+        lib.cbo_score_self.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_double, ctypes.c_double,
+                                       ctypes.c_double, ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P, _P, _P]
+        lib.cbo_score_self.restype = ctypes.c_int
+        lib.cbo_attention_self.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_double, _P]
+        lib.cbo_attention_self.restype = ctypes.c_int
         for name, ptr_t in (("cbo_select_f64", _P), ("cbo_select_f32", _P)):
             f = getattr(lib, name)
             f.argtypes = [ctypes.c_int64, ptr_t, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
@@ -108,27 +114,43 @@ class Oracle:
         return int(self.lib.cbo_max_threads())
 
     # -- App. C.1 ------------------------------------------------------------
+    def _self_keys(self, dm: _Dims, Kself):
+        """Bits of the query's own keys [nL][m][Hkv][d] (or None) with their strides set in dm."""
+        if Kself is None:
+            return None
+        Ksb = self._bits(Kself)
+        if Ksb.shape != (dm.n_layers, dm.m, dm.n_kv_heads, dm.head_dim):
+            raise ValueError("the query's own keys must be [nL][m][Hkv][d]")
+        dm.s_layer, dm.s_tok, dm.s_head = dm.m * dm.n_kv_heads * dm.head_dim, dm.n_kv_heads * dm.head_dim, dm.head_dim
+        return Ksb
+
     def score(self, K, Q, p: float = 2.0, alpha: float = 2.0, pool_w: int = 7,
-              scale: Optional[float] = None, n_threads: int = 0) -> dict:
+              scale: Optional[float] = None, n_threads: int = 0, Kself=None) -> dict:
+        """Kself: the query tokens' own keys [nL][m][Hkv][d]; each query token's softmax then
+        also runs over the keys of query tokens 0..r (None: sender positions only)."""
         Kb, Qb = self._bits(K), self._bits(Q)
         dm = self._dims(Kb, Qb)
+        Ksb = self._self_keys(dm, Kself)
         T = dm.T
         if scale is None:
             scale = 1.0 / math.sqrt(dm.head_dim)
         out = {k: np.zeros(T, dtype=np.float64) for k in ("S", "Q", "C", "U", "N", "D")}
-        st = self.lib.cbo_score(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data, scale, p, alpha,
-                                pool_w, n_threads, *(out[k].ctypes.data for k in ("S", "Q", "C", "U", "N", "D")))
+        st = self.lib.cbo_score_self(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data,
+                                     None if Ksb is None else Ksb.ctypes.data, scale, p, alpha, pool_w, n_threads,
+                                     *(out[k].ctypes.data for k in ("S", "Q", "C", "U", "N", "D")))
         if st != OK:
             raise RuntimeError("cbo_score failed with status %d" % st)
         return out
 
-    def attention(self, K, Q, scale: Optional[float] = None) -> np.ndarray:
+    def attention(self, K, Q, scale: Optional[float] = None, Kself=None) -> np.ndarray:
         Kb, Qb = self._bits(K), self._bits(Q)
         dm = self._dims(Kb, Qb)
+        Ksb = self._self_keys(dm, Kself)
         if scale is None:
             scale = 1.0 / math.sqrt(dm.head_dim)
         a = np.zeros((dm.n_layers, dm.n_q_heads, dm.m, dm.T), dtype=np.float64)
-        st = self.lib.cbo_attention(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data, scale, a.ctypes.data)
+        st = self.lib.cbo_attention_self(ctypes.byref(dm), Kb.ctypes.data, Qb.ctypes.data,
+                                         None if Ksb is None else Ksb.ctypes.data, scale, a.ctypes.data)
         if st != OK:
             raise RuntimeError("cbo_attention failed with status %d" % st)
         return a

@@ -27,26 +27,34 @@ def pool(x: np.ndarray, w: int = 7) -> np.ndarray:
     return out
 
 
-def attention(Kd: np.ndarray, Qd: np.ndarray, scale: float) -> np.ndarray:
-    """a[l][h][r][t] with query head h reading KV head h // G."""
+def attention(Kd: np.ndarray, Qd: np.ndarray, scale: float, Ksd=None) -> np.ndarray:
+    """a[l][h][r][t] with query head h reading KV head h // G.  Ksd [nL][m][Hkv][d]: the query
+    tokens' own keys, appended to every row's softmax with a causal mask (token r sees 0..r);
+    only the sender columns are returned."""
     nL, Hkv, T, d = Kd.shape
     _, m, Hq, _ = Qd.shape
     G = Hq // Hkv
     Krep = np.repeat(Kd, G, axis=1)                      # [nL][Hq][T][d]
     z = np.einsum("lrhd,lhtd->lhrt", Qd, Krep) * scale   # [nL][Hq][m][T]
+    if Ksd is not None:
+        Ksrep = np.repeat(Ksd, G, axis=2)                # [nL][m][Hq][d]
+        zs = np.einsum("lrhd,luhd->lhru", Qd, Ksrep) * scale   # [nL][Hq][m][m]
+        causal = np.tril(np.ones((m, m), dtype=bool))
+        zs = np.where(causal, zs, -np.inf)
+        z = np.concatenate([z, zs], axis=-1)
     z = z - z.max(axis=-1, keepdims=True)
     e = np.exp(z)
-    return e / e.sum(axis=-1, keepdims=True)
+    return (e / e.sum(axis=-1, keepdims=True))[..., :T]
 
 
-def score(Kbits, Qbits, p=2.0, alpha=2.0, pool_w=7, scale=None) -> dict:
+def score(Kbits, Qbits, p=2.0, alpha=2.0, pool_w=7, scale=None, Ksbits=None) -> dict:
     Kd, Qd = bf16_bits_to_f64(Kbits), bf16_bits_to_f64(Qbits)
     nL, Hkv, T, d = Kd.shape
     _, m, Hq, _ = Qd.shape
     G = Hq // Hkv
     if scale is None:
         scale = 1.0 / math.sqrt(d)
-    a = attention(Kd, Qd, scale)
+    a = attention(Kd, Qd, scale, None if Ksbits is None else bf16_bits_to_f64(Ksbits))
     # mean query attention: sum over layers of the (r, h)-average, then Pool
     U = a.mean(axis=(1, 2)).sum(axis=0)                  # [T]
     Qt = pool(U, pool_w)

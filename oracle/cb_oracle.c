@@ -48,6 +48,7 @@ typedef struct {
     int64_t T;          /* sender positions */
     int64_t k_layer, k_head, k_pos; /* element strides of K and V, dim stride 1 */
     int64_t q_layer, q_tok, q_head; /* element strides of Q, dim stride 1 */
+    int64_t s_layer, s_tok, s_head; /* element strides of the query's own keys Ks[l][u][g][:], if given */
 } cbo_dims;
 
 /* bf16 bit pattern -> double, exact. */
@@ -96,14 +97,26 @@ static double *load_keys_transposed(const cbo_dims *dm, const uint16_t *K, int l
     return kt;
 }
 
+/* scale * <q, ks_{l,u,g}>: logit of a query token against query token u's own key. */
+static double self_logit(const cbo_dims *dm, const uint16_t *q, const uint16_t *Ks, int l, int u, int g,
+                         double scale) {
+    const uint16_t *k = Ks + (int64_t)l * dm->s_layer + (int64_t)u * dm->s_tok + (int64_t)g * dm->s_head;
+    double z = 0.0;
+    for (int i = 0; i < dm->head_dim; ++i) z += bf16_to_double(q[i]) * bf16_to_double(k[i]);
+    return z * scale;
+}
+
 /*
  * One attention row a_{l,h,r,.} (App. C.1, "Adapting SnapKV"): the sender
  * attends from query token r, head h, to its cached positions:
  *   z_t = scale * <q_{l,r,h}, k_{l,g(h),t}>,   a_t = exp(z_t - M) / sum_u exp(z_u - M),
  * with M = max_t z_t (the shift leaves a unchanged).  z is scratch of length T.
+ * With the query tokens' own keys Ks (not NULL) the softmax also runs over the keys of query
+ * tokens 0..r (the causal prefix of the query in a real forward pass); a still covers the
+ * sender positions only, so it sums to less than one.
  */
-static void attention_row(const cbo_dims *dm, const double *kt, const uint16_t *Q, int l, int h, int r,
-                          double scale, double *z, double *a) {
+static void attention_row(const cbo_dims *dm, const double *kt, const uint16_t *Q, const uint16_t *Ks, int l,
+                          int h, int r, double scale, double *z, double *a) {
     int64_t T = dm->T;
     int d = dm->head_dim;
     const uint16_t *q = Q + (int64_t)l * dm->q_layer + (int64_t)r * dm->q_tok + (int64_t)h * dm->q_head;
@@ -118,11 +131,19 @@ static void attention_row(const cbo_dims *dm, const double *kt, const uint16_t *
         z[t] *= scale;
         if (z[t] > M) M = z[t];
     }
+    const int g = h / (dm->n_q_heads / dm->n_kv_heads);
+    if (Ks)
+        for (int u = 0; u <= r; ++u) {
+            const double zs = self_logit(dm, q, Ks, l, u, g, scale);
+            if (zs > M) M = zs;
+        }
     double Z = 0.0;
     for (int64_t t = 0; t < T; ++t) {
         a[t] = exp(z[t] - M);
         Z += a[t];
     }
+    if (Ks)
+        for (int u = 0; u <= r; ++u) Z += exp(self_logit(dm, q, Ks, l, u, g, scale) - M);
     for (int64_t t = 0; t < T; ++t) a[t] /= Z;
 }
 
@@ -131,7 +152,8 @@ static void attention_row(const cbo_dims *dm, const double *kt, const uint16_t *
  * Exposed so tests can check the softmax and the head-to-KV-head mapping
  * against a library attention routine.
  */
-int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double scale, double *a) {
+int cbo_attention_self(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, const uint16_t *Ks, double scale,
+                       double *a) {
     int st = check_dims(dm);
     if (st) return st;
     if (!K || !Q || !a) return CBO_EINVAL;
@@ -144,7 +166,7 @@ int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, doub
             double *kt = load_keys_transposed(dm, K, l, h / G);
             if (!kt) { free(z); return CBO_ENOMEM; }
             for (int r = 0; r < dm->m; ++r)
-                attention_row(dm, kt, Q, l, h, r, scale,
+                attention_row(dm, kt, Q, Ks, l, h, r, scale,
                               z, a + (((int64_t)l * dm->n_q_heads + h) * dm->m + r) * T);
             free(kt);
         }
@@ -152,8 +174,13 @@ int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, doub
     return CBO_OK;
 }
 
+int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double scale, double *a) {
+    return cbo_attention_self(dm, K, Q, NULL, scale, a);
+}
+
 /*
- * Score every sender position (App. C.1 and App. D.2):
+ * Score every sender position (App. C.1 and App. D.2); Ks (may be NULL) are the query tokens'
+ * own keys, joining each query token's softmax causally (see attention_row):
  *
  *   Q_t   = Pool( sum_l 1/(m |H_l|) sum_r sum_{h in H_l} a_{l,h,r,t} )          (mean query attention)
  *   C_p,t = ( sum_s mean_r[Pool(b_{s,r,.})_t^p] / sum_s Pool(mean_r b_{s,r,.})_t^p )^(1/(p-1))
@@ -169,9 +196,9 @@ int cbo_attention(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, doub
  * The work is split over the groups s = (l, g); each group's contributions are
  * kept apart and added in the order s = 0, 1, ... at the end.
  */
-int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double scale, double p,
-              double alpha, int32_t pool_w, int32_t n_threads, double *S, double *Qt, double *C, double *U,
-              double *N, double *D) {
+int cbo_score_self(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, const uint16_t *Ks, double scale,
+                   double p, double alpha, int32_t pool_w, int32_t n_threads, double *S, double *Qt, double *C,
+                   double *U, double *N, double *D) {
     int st = check_dims(dm);
     if (st) return st;
     if (!K || !Q) return CBO_EINVAL;
@@ -205,7 +232,7 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
                 double *br = b + (int64_t)r * T;
                 for (int j = 0; j < G; ++j) {
                     const int h = g * G + j;
-                    attention_row(dm, kt, Q, l, h, r, scale, z, a);
+                    attention_row(dm, kt, Q, Ks, l, h, r, scale, z, a);
                     for (int64_t t = 0; t < T; ++t) {
                         br[t] += a[t] / G;                 /* b_{s,r,t}: mean over the group's heads */
                         Us[t] += a[t] / ((double)m * Hq);  /* this group's share of the layer term of Q_t */
@@ -265,6 +292,11 @@ int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double s
     }
     free(part); free(Usum); free(Nsum); free(Dsum); free(Qv);
     return CBO_OK;
+}
+
+int cbo_score(const cbo_dims *dm, const uint16_t *K, const uint16_t *Q, double scale, double p, double alpha,
+              int32_t pool_w, int32_t n_threads, double *S, double *Qt, double *C, double *U, double *N, double *D) {
+    return cbo_score_self(dm, K, Q, NULL, scale, p, alpha, pool_w, n_threads, S, Qt, C, U, N, D);
 }
 
 /* ---------------------------------------------------------------------------

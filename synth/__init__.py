@@ -228,6 +228,13 @@ def make_query(spec: WorkloadSpec, seed: int, task: int, device="cpu") -> torch.
     return normal_bf16_shaped((s.n_layers, spec.m, s.n_q_heads, s.head_dim), key, device)
 
 
+def make_query_keys(spec: WorkloadSpec, seed: int, task: int, device="cpu") -> torch.Tensor:
+    """The receiver query tokens' own post-RoPE keys, bf16 [nL][m][Hkv][d], N(0,1)."""
+    s = spec.shape
+    key = stream_key(seed, 7, task)          # a stream of its own (K and V use ids 2 and 3)
+    return normal_bf16_shaped((s.n_layers, spec.m, s.n_kv_heads, s.head_dim), key, device)
+
+
 def _directions(spec: WorkloadSpec, Qcpu: torch.Tensor, rng: np.random.Generator) -> torch.Tensor:
     """Per-(layer, KV head) unit-RMS direction taken from one query row (fp32, CPU)."""
     s = spec.shape

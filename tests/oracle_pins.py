@@ -279,6 +279,30 @@ def pin_p_infinity(o):
     assert np.allclose(o.score(K, Q[:, :1].contiguous(), p=inf)["C"], 1.0, rtol=1e-13, atol=0)
 
 
+def pin_self_keys(o):
+    """The query tokens' own keys in the softmax (the causal prefix of a real forward pass): the
+    sender attention equals torch's SDPA over [sender keys, query keys] with query token r
+    allowed the query keys 0..r, and the scores equal the numpy restatement."""
+    nL, Hq, Hkv, d, T, m = 2, 8, 2, 16, 37, 5
+    K, _, Q = _rand_case(nL, Hq, Hkv, d, T, m, seed=41)
+    Ks = synth.normal_bf16_shaped((nL, m, Hkv, d), synth.stream_key(41, 99))
+    a = o.attention(K, Q, Kself=Ks)
+    G = Hq // Hkv
+    Kall = torch.cat([K.to(torch.float64), Ks.to(torch.float64).permute(0, 2, 1, 3)], dim=2)   # [nL][Hkv][T+m][d]
+    Kall = Kall.repeat_interleave(G, dim=1)                                                   # [nL][Hq][T+m][d]
+    Qd = Q.to(torch.float64).permute(0, 2, 1, 3)                                              # [nL][Hq][m][d]
+    mask = torch.ones(m, T + m, dtype=torch.bool)
+    mask[:, T:] = torch.tril(torch.ones(m, m, dtype=torch.bool))
+    eye = torch.eye(T + m, dtype=torch.float64).expand(nL, Hq, T + m, T + m)
+    ref = torch.nn.functional.scaled_dot_product_attention(Qd, Kall, eye, attn_mask=mask, scale=d ** -0.5)
+    assert _rel(a, ref[..., :T].numpy()) < 1e-12
+    assert np.all(a.sum(axis=-1) < 1.0)                  # part of every row's mass is on query keys
+    r = o.score(K, Q, Kself=Ks)
+    b = brute.score(_bits(K), _bits(Q), Ksbits=_bits(Ks))
+    for k in ("S", "Q", "C", "U", "N", "D"):
+        assert _rel(r[k], b[k]) < 1e-12, (k, _rel(r[k], b[k]))
+
+
 # --------------------------------------------------------------------------
 # selection (App. C.2)
 # --------------------------------------------------------------------------
@@ -355,6 +379,7 @@ def pin_gather(o):
 ALL_PINS = [
     pin_pool_one_hot, pin_pool_library, pin_attention_sdpa, pin_one_hot_closed_form,
     pin_zero_denominator, pin_variance_identity, pin_identical_keys, pin_invariants,
-    pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_select_golden, pin_select_integrity,
+    pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_self_keys, pin_select_golden,
+    pin_select_integrity,
     pin_compact, pin_gather,
 ]

@@ -56,6 +56,9 @@ MUTANTS = [
     ("compact_offset_dropped", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + (off + j) * d;", "int64_t dst = (int64_t)l * o_layer + (int64_t)g * o_head + j * d;"),
     ("gather_offset_dropped", "memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);", "memcpy(out + j * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);"),
     ("gather_row_shifted", "memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);", "memcpy(out + (off + j) * out_stride, src + (int64_t)(idx[j] + (idx[j] + 1 < T)) * src_stride, (size_t)row_bytes);"),
+    ("self_keys_not_causal", "for (int u = 0; u <= r; ++u) Z += exp(", "for (int u = 0; u < dm->m; ++u) Z += exp("),
+    ("self_keys_unscaled", "    return z * scale;\n}", "    return z;\n}"),
+    ("self_keys_wrong_group", "(int64_t)g * dm->s_head;", "(int64_t)((g + 1) % dm->n_kv_heads) * dm->s_head;"),
     ("compact_v_from_k", "memcpy(v_out + dst, V + src, sizeof(uint16_t) * (size_t)d);", "memcpy(v_out + dst, K + src, sizeof(uint16_t) * (size_t)d);"),
 ]
 
