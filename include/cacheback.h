@@ -97,11 +97,19 @@ typedef struct {
 
 /* The receiver query's post-RoPE query vectors in the sender's scored layers (Sec. 3:
  * the sender appends q and computes only the query tokens against its cache):
- * Q[l][r][h][:] at q + l*s_layer + r*s_tok + h*s_head, r < m.  Several senders may share one. */
+ * Q[l][r][h][:] at q + l*s_layer + r*s_tok + h*s_head, r < m.  Several senders may share one.
+ * k_self (optional, NULL for none): the query tokens' own post-RoPE keys, Ks[l][u][g][:] at
+ * k_self + l*ks_layer + u*ks_tok + g*ks_head (u < m, g < Hkv; strides positive multiples of 8).
+ * When given, query token r's softmax also runs over the keys of query tokens 0..r, as the
+ * appended query attends causally in a real forward pass; the scores still cover the sender
+ * positions only, whose attention then sums to less than one.  NULL keeps App. C.1's reading:
+ * the softmax over the T sender positions. */
 typedef struct {
     const void *q;
     int32_t m;
     int64_t s_layer, s_tok, s_head;
+    const void *k_self;
+    int64_t ks_layer, ks_tok, ks_head;
 } cb_query;
 
 /* Fill *cfg with the paper's defaults (p = alpha = 2, Pool_7, width-16 spans, 1 sink,

@@ -29,12 +29,15 @@ class Filter:
     The send buffer holds every sender's rows back to back: sender i at offset sum_{j<i} B_j.
     """
 
-    def __init__(self, cb: CacheBack, senders: Sequence, queries: Sequence, keep: float, device=None):
+    def __init__(self, cb: CacheBack, senders: Sequence, queries: Sequence, keep: float, device=None,
+                 query_keys: Optional[Sequence] = None):
         import torch
         self.cb = cb
         self.Ks = [k for k, _ in senders]
         self.Vs = [v for _, v in senders]
         self.Qs = list(queries)
+        # optional: the query tokens' own keys [nL][m][Hkv][d] per sender (None: sender positions only)
+        self.Kqs = list(query_keys) if query_keys is not None else [None] * len(self.Ks)
         dev = device or self.Ks[0].device
         self.Ts = [int(K.shape[2]) for K in self.Ks]
         # B_i = ceil(keep * T_i), raised to the forced count when that is larger (App. C.2: the
@@ -54,7 +57,7 @@ class Filter:
         self.v_out = torch.empty_like(self.k_out)
 
     def score(self, stream=None):
-        self.cb.score(self.Ks, self.Qs, self.scores, stream)
+        self.cb.score(self.Ks, self.Qs, self.scores, stream, self.Kqs)
 
     def select(self, stream=None):
         self.cb.select(self.scores, self.Ts, self.budgets, self.idx, stream)
@@ -81,7 +84,7 @@ class Filter:
         for a in range(0, n, wave):
             b = min(n, a + wave)
             sl = slice(a, b)
-            self.cb.score(self.Ks[sl], self.Qs[sl], self.scores[sl], main)
+            self.cb.score(self.Ks[sl], self.Qs[sl], self.scores[sl], main, self.Kqs[sl])
             done = torch.cuda.Event()
             done.record(main)
             side.wait_event(done)

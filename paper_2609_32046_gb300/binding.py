@@ -48,7 +48,8 @@ class cb_kv(ctypes.Structure):
 
 class cb_query(ctypes.Structure):
     _fields_ = [("q", ctypes.c_void_p), ("m", ctypes.c_int32), ("s_layer", ctypes.c_int64),
-                ("s_tok", ctypes.c_int64), ("s_head", ctypes.c_int64)]
+                ("s_tok", ctypes.c_int64), ("s_head", ctypes.c_int64), ("k_self", ctypes.c_void_p),
+                ("ks_layer", ctypes.c_int64), ("ks_tok", ctypes.c_int64), ("ks_head", ctypes.c_int64)]
 
 
 _LIB = None
@@ -156,10 +157,14 @@ def kv_desc(K, V=None) -> cb_kv:
                  K.stride(0), K.stride(1), K.stride(2))
 
 
-def query_desc(Q) -> cb_query:
-    """Q: bf16 [nL][m][Hq][d]."""
+def query_desc(Q, Kself=None) -> cb_query:
+    """Q: bf16 [nL][m][Hq][d]; Kself (optional): the query tokens' own keys, bf16 [nL][m][Hkv][d]."""
     assert Q.dtype.itemsize == 2 and Q.stride(3) == 1
-    return cb_query(Q.data_ptr(), Q.shape[1], Q.stride(0), Q.stride(1), Q.stride(2))
+    if Kself is None:
+        return cb_query(Q.data_ptr(), Q.shape[1], Q.stride(0), Q.stride(1), Q.stride(2), None, 0, 0, 0)
+    assert Kself.dtype.itemsize == 2 and Kself.stride(3) == 1 and Kself.shape[1] == Q.shape[1]
+    return cb_query(Q.data_ptr(), Q.shape[1], Q.stride(0), Q.stride(1), Q.stride(2), Kself.data_ptr(),
+                    Kself.stride(0), Kself.stride(1), Kself.stride(2))
 
 
 class CacheBack:
@@ -208,10 +213,13 @@ class CacheBack:
         return int(self.lib.cb_score_path(self.h))
 
     # -- the three steps ----------------------------------------------------
-    def score(self, Ks: Sequence, Qs: Sequence, scores: Sequence, stream=None):
+    def score(self, Ks: Sequence, Qs: Sequence, scores: Sequence, stream=None, Kselfs: Optional[Sequence] = None):
+        """Kselfs (optional): per sender, the query tokens' own keys (or None) that join each
+        query token's softmax causally."""
         n = len(Ks)
         kv = (cb_kv * n)(*[kv_desc(K) for K in Ks])
-        qq = (cb_query * n)(*[query_desc(Q) for Q in Qs])
+        Kselfs = Kselfs or [None] * n
+        qq = (cb_query * n)(*[query_desc(Q, Kq) for Q, Kq in zip(Qs, Kselfs)])
         out = _ptr_array([s.data_ptr() for s in scores])
         self._check(self.lib.cb_score(self.h, n, kv, qq, out, _stream_handle(stream)))
 

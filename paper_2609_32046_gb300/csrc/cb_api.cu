@@ -297,6 +297,12 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         cb_status st;
         if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
         if ((st = check_device_ptr(ctx, q.q, "queries.q", i))) return st;
+        if (q.k_self) {
+            if (!stride_ok(q.ks_layer) || !stride_ok(q.ks_tok) || !stride_ok(q.ks_head) || q.ks_head < c.head_dim)
+                return fail(ctx, CB_EINVAL, "queries[%d]: k_self strides must be positive multiples of 8 "
+                            "(ks_head >= d)", i);
+            if ((st = check_device_ptr(ctx, q.k_self, "queries.k_self", i))) return st;
+        }
         if ((st = check_device_ptr(ctx, scores[i], "scores", i))) return st;
     }
     cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
@@ -334,6 +340,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.T = s.T;
             d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
             d.qs_l = q.s_layer; d.qs_t = q.s_tok; d.qs_h = q.s_head;
+            d.kself = static_cast<const uint16_t*>(q.k_self);
+            d.kss_l = q.ks_layer; d.kss_t = q.ks_tok; d.kss_h = q.ks_head;
             d.m = q.m;
             d.n_chunk1 = (int32_t)((s.T + cbk::kStatsChunk - 1) / cbk::kStatsChunk);
             d.n_chunk2 = (int32_t)((s.T + cbk::kAccumChunk - 1) / cbk::kAccumChunk);

@@ -43,6 +43,8 @@ struct ScoreSender {
     int64_t T;
     int64_t ks_l, ks_h, ks_p;
     int64_t qs_l, qs_t, qs_h;
+    const uint16_t* kself;    // the query tokens' own keys Ks[l][u][g][:] or null
+    int64_t kss_l, kss_t, kss_h;
     int32_t m;
     int32_t n_chunk1;         // ceil(T / kStatsChunk)
     int32_t n_chunk2;         // ceil(T / kAccumChunk)

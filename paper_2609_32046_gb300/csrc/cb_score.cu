@@ -284,6 +284,34 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
                 L += v.y * ex2(v.x - M);
             }
         }
+        if (sd.kself) {
+            // the query tokens' own keys: row (token r, head h) also attends to query keys
+            // 0..r (every fourth one on this slot lane); logits in the statistics' log2 domain
+            const int r = row / G, hh = row - r * G;
+            const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
+            const uint16_t* qrow = sd.q + (int64_t)l * sd.qs_l + (int64_t)r * sd.qs_t + (int64_t)(g * G + hh) * sd.qs_h;
+            for (int u = j; u <= r; u += 4) {
+                const uint16_t* krow = sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h;
+                float dot = 0.f;
+                for (int k = 0; k < bt.head_dim; k += 8) {
+                    const uint4 a = *reinterpret_cast<const uint4*>(qrow + k);
+                    const uint4 b = *reinterpret_cast<const uint4*>(krow + k);
+                    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        dot = fmaf(__uint_as_float(aw[w] << 16), __uint_as_float(bw[w] << 16), dot);
+                        dot = fmaf(__uint_as_float(aw[w] & 0xFFFF0000u), __uint_as_float(bw[w] & 0xFFFF0000u), dot);
+                    }
+                }
+                const float x = dot * bt.scale_log2e;
+                if (x > M) {
+                    L = (M == -INFINITY ? 0.f : L * ex2(M - x)) + 1.f;
+                    M = x;
+                } else {
+                    L += ex2(x - M);
+                }
+            }
+        }
     }
     part[j][threadIdx.x & (kCombRows - 1)] = make_float2(M, L);
     __syncthreads();

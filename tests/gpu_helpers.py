@@ -27,22 +27,25 @@ def make_cb(shape, max_positions, m, n_senders=1, **kw):
                         max_positions, n_senders, **kw)
 
 
-def run_path(workload, keep, device="cuda", **kw):
-    """CUDA path over every sender of the workload: returns the Filter (results on device)."""
+def run_path(workload, keep, device="cuda", query_keys=None, **kw):
+    """CUDA path over every sender of the workload: returns the Filter (results on device).
+    query_keys: optional per-sender query self-keys (joining the softmax causally)."""
     spec = workload.spec
     senders = [(s.K.to(device), s.V.to(device)) for s in workload.senders]
     queries = [workload.queries[s.task].to(device) for s in workload.senders]
     m = max(q.shape[1] for q in queries)
     c = make_cb(spec.shape, max(s.T for s in workload.senders), m, len(senders), **kw)
-    f = cb.Filter(c, senders, queries, keep)
+    qk = None if query_keys is None else [k.to(device) for k in query_keys]
+    f = cb.Filter(c, senders, queries, keep, query_keys=qk)
     f.run()
     c.sync_status()
     torch.cuda.synchronize()
     return f
 
 
-def oracle_scores(o, K, Q, p=2.0, alpha=2.0, pool_w=7, scale=None):
-    return o.score(K.cpu(), Q.cpu(), p=p, alpha=alpha, pool_w=pool_w, scale=scale)
+def oracle_scores(o, K, Q, p=2.0, alpha=2.0, pool_w=7, scale=None, Kself=None):
+    return o.score(K.cpu(), Q.cpu(), p=p, alpha=alpha, pool_w=pool_w, scale=scale,
+                   Kself=None if Kself is None else Kself.cpu())
 
 
 def assert_scores_close(gpu_S, ref_S, rtol=SCORE_RTOL):
@@ -97,10 +100,10 @@ def assert_compact_exact(f, sender_index, K, V, idx):
 
 
 def check_sender(f, i, K, V, Q, o=None, p=2.0, alpha=2.0, pool_w=7, span_w=16, n_sink=1, n_latent=40,
-                 scale=None):
+                 scale=None, Kself=None):
     """Full parity of sender i of a finished Filter run against the oracle."""
     o = o or oracle.default()
-    ref = oracle_scores(o, K, Q, p=p, alpha=alpha, pool_w=pool_w, scale=scale)
+    ref = oracle_scores(o, K, Q, p=p, alpha=alpha, pool_w=pool_w, scale=scale, Kself=Kself)
     gS = f.scores[i].cpu().numpy()
     err = assert_scores_close(gS, ref["S"])
     B = f.budgets[i]

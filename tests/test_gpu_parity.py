@@ -40,6 +40,10 @@ CASES = [
     ("p_inf_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(p=float("inf"))),
     ("p_inf_g2_pool5", (2, 8, 4, 128), [611], 20, 0.3, dict(p=float("inf"), pool_width=5, alpha=3.0)),
     ("p_inf_d64", (2, 8, 2, 64), [600], 12, 0.2, dict(p=float("inf"))),
+    # the query tokens' own keys join the softmax causally
+    ("self_keys_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(self_keys=True)),
+    ("self_keys_g2_d64", (2, 8, 4, 64), [333], 17, 0.3, dict(self_keys=True)),
+    ("self_keys_fan_in_m128", (1, 16, 4, 128), [300, 129], 128, 0.25, dict(self_keys=True)),
     # more senders than one tcgen05 launch takes (32): two launches per pass
     ("forty_senders", (1, 8, 2, 128), [97 + 13 * i for i in range(40)], 8, 0.3, {}),
 ]
@@ -65,12 +69,16 @@ def test_parity(case, kernel):
     if kernel == 2 and not _tc_supported(shape, m, extra):
         pytest.skip("shape outside the tcgen05 score path")
     w = _workload(name, shape, Ts, m)
-    f = run_path(w, keep, score_kernel=kernel, **extra)
+    extra = dict(extra)
+    qk = None
+    if extra.pop("self_keys", False):
+        qk = [synth.make_query_keys(w.spec, 5, s.task) for s in w.senders]
+    f = run_path(w, keep, score_kernel=kernel, query_keys=qk, **extra)
     assert f.cb.score_path() == kernel, "the requested logit-pass kernels did not run"
     kw = dict(p=extra.get("p", 2.0), alpha=extra.get("alpha", 2.0), pool_w=extra.get("pool_width", 7),
               span_w=extra.get("span_width", 16))
     for i, s in enumerate(w.senders):
-        check_sender(f, i, s.K, s.V, w.queries[s.task], **kw)
+        check_sender(f, i, s.K, s.V, w.queries[s.task], Kself=None if qk is None else qk[i], **kw)
 
 
 def test_select_on_oracle_scores_is_exact():
