@@ -79,6 +79,10 @@ class Oracle:
         lib.cbo_compact.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_int64, _P, _P,
                                     ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
         lib.cbo_compact.restype = ctypes.c_int
+        lib.cbo_compact_rope.argtypes = [ctypes.POINTER(_Dims), _P, _P, _P, ctypes.c_int64, _P, _P, ctypes.c_int64,
+                                         ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.c_int32,
+                                         ctypes.c_int64]
+        lib.cbo_compact_rope.restype = ctypes.c_int
         lib.cbo_gather.argtypes = [_P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, _P, ctypes.c_int64, _P,
                                    ctypes.c_int64, ctypes.c_int64]
         lib.cbo_gather.restype = ctypes.c_int
@@ -193,6 +197,26 @@ class Oracle:
             raise RuntimeError("cbo_compact failed with status %d" % st)
         return out_k, out_v
 
+
+    def compact_rope(self, K, V, idx, base: float, style: int = 0, pos0: int = 0, out_k=None, out_v=None,
+                     offset: int = 0):
+        """Compaction with K moved from its sender positions idx[j] to receiver positions
+        pos0 + offset + j by the rotary embedding (style 0: halves, 1: interleaved pairs)."""
+        Kb, Vb = self._bits(K), self._bits(V)
+        nL, Hkv, T, d = Kb.shape
+        idx = np.ascontiguousarray(idx, dtype=np.int32)
+        B = idx.shape[0]
+        if out_k is None:
+            out_k = np.zeros((nL, Hkv, offset + B, d), dtype=np.uint16)
+            out_v = np.zeros_like(out_k)
+        cap = out_k.shape[2]
+        dm = _Dims(nL, Hkv, Hkv, d, 1, T, Hkv * T * d, T * d, d, 0, 0, 0)
+        st = self.lib.cbo_compact_rope(ctypes.byref(dm), Kb.ctypes.data, Vb.ctypes.data, idx.ctypes.data, B,
+                                       out_k.ctypes.data, out_v.ctypes.data, offset, Hkv * cap * d, cap * d,
+                                       base, style, pos0)
+        if st != OK:
+            raise RuntimeError("cbo_compact_rope failed with status %d" % st)
+        return out_k, out_v
 
     def gather(self, table, idx, out=None, offset: int = 0) -> np.ndarray:
         """Message rows (App. C.3): out[offset + j] = table[idx[j]] as raw bytes.  table: numpy

@@ -465,4 +465,55 @@ int cbo_gather(const uint8_t *src, int64_t T, int64_t src_stride, int64_t row_by
     return CBO_OK;
 }
 
+/* double -> bf16 bits, rounded once to nearest (ties to even); finite normal inputs. */
+static uint16_t double_to_bf16(double x) {
+    if (x == 0.0) return signbit(x) ? 0x8000u : 0u;
+    int e;
+    const double m = frexp(x, &e);                 /* |m| in [0.5, 1) */
+    const double r = nearbyint(ldexp(m, 8));       /* 8 significant bits, ties to even */
+    const float f = (float)ldexp(r, e - 8);         /* exact: a bf16 value */
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    return (uint16_t)(u >> 16);
+}
+
+/*
+ * Compaction with the positional re-index direct K/V transfer needs (App. C.3: a receiver that
+ * takes the sender's K rows as they are must move them from sender position t to its own
+ * position p).  Rotary embeddings rotate each pair of K's dimensions by angle pos * theta_k with
+ * theta_k = base^(-2k/d), k < d/2, so a row rotated for t becomes the row for p by one more
+ * rotation by (p - t) * theta_k:
+ *   (x_a, x_b) -> (x_a cos phi - x_b sin phi, x_b cos phi + x_a sin phi),  phi = (p - t) theta_k,
+ * pairs (a, b) = (k, k + d/2) for style 0 (halves) or (2k, 2k + 1) for style 1 (interleaved).
+ * Row j of the output (at out offset off) sits at receiver position p = pos0 + off + j.
+ * K is rotated in double and rounded once to bf16; V is copied as in cbo_compact.
+ */
+int cbo_compact_rope(const cbo_dims *dm, const uint16_t *K, const uint16_t *V, const int32_t *idx, int64_t B,
+                     uint16_t *k_out, uint16_t *v_out, int64_t off, int64_t o_layer, int64_t o_head, double base,
+                     int32_t style, int64_t pos0) {
+    int st = check_dims(dm);
+    if (st) return st;
+    if (!K || !V || !idx || !k_out || !v_out || B < 0 || !(base > 0.0) || (style != 0 && style != 1)) return CBO_EINVAL;
+    const int d = dm->head_dim, half = d / 2;
+    if (d % 2) return CBO_ESHAPE;
+    for (int64_t j = 0; j < B; ++j)
+        if (idx[j] < 0 || idx[j] >= dm->T) return CBO_EINVAL;
+    for (int l = 0; l < dm->n_layers; ++l)
+        for (int g = 0; g < dm->n_kv_heads; ++g)
+            for (int64_t j = 0; j < B; ++j) {
+                const int64_t src = (int64_t)l * dm->k_layer + (int64_t)g * dm->k_head + (int64_t)idx[j] * dm->k_pos;
+                const int64_t dst = (off + j) * d + (int64_t)g * o_head + (int64_t)l * o_layer;
+                const double delta = (double)(pos0 + off + j - idx[j]);
+                for (int k = 0; k < half; ++k) {
+                    const int a = style == 0 ? k : 2 * k, b = style == 0 ? k + half : 2 * k + 1;
+                    const double phi = delta * pow(base, -2.0 * k / d);
+                    const double xa = bf16_to_double(K[src + a]), xb = bf16_to_double(K[src + b]);
+                    k_out[dst + a] = double_to_bf16(xa * cos(phi) - xb * sin(phi));
+                    k_out[dst + b] = double_to_bf16(xb * cos(phi) + xa * sin(phi));
+                }
+                memcpy(&v_out[dst], &V[src], sizeof(uint16_t) * (size_t)d);
+            }
+    return CBO_OK;
+}
+
 int cbo_max_threads(void) { return omp_get_max_threads(); }

@@ -365,6 +365,47 @@ def pin_compact(o):
     assert not ko[:, :, :off].any() and not vo[:, :, :off].any()
 
 
+def _rope_ref(x, pos, base, style):
+    """Textbook rotary embedding of x [..., d] at integer positions pos [...] (float64 torch)."""
+    d = x.shape[-1]
+    theta = base ** (-2.0 * torch.arange(d // 2, dtype=torch.float64) / d)
+    ang = pos.to(torch.float64)[..., None] * theta
+    c, s = torch.cos(ang), torch.sin(ang)
+    if style == 0:                                        # rotate_half: pairs (k, k + d/2)
+        x1, x2 = x[..., : d // 2], x[..., d // 2:]
+        return torch.cat([x1 * c - x2 * s, x2 * c + x1 * s], dim=-1)
+    xe, xo = x[..., 0::2], x[..., 1::2]                   # interleaved pairs (2k, 2k + 1)
+    out = torch.empty_like(x)
+    out[..., 0::2] = xe * c - xo * s
+    out[..., 1::2] = xo * c + xe * s
+    return out
+
+
+def pin_compact_rope(o):
+    """K moved from sender positions to receiver positions: equals the textbook rotary embedding
+    applied at the new positions to the raw keys (within the two bf16 roundings), is the identity
+    when the positions agree, keeps V unchanged."""
+    nL, Hkv, T, d, base = 2, 2, 90, 32, 10000.0
+    g = torch.Generator().manual_seed(8)
+    raw = torch.randn(nL, Hkv, T, d, generator=g, dtype=torch.float64)
+    pos = torch.arange(T)
+    V = torch.randn(nL, Hkv, T, d, generator=g).to(torch.bfloat16)
+    idx = np.array([0, 5, 6, 30, 61, 89], dtype=np.int32)
+    for style in (0, 1):
+        K = _rope_ref(raw, pos.expand(nL, Hkv, T), base, style).to(torch.bfloat16)
+        pos0, off = 1000, 3
+        ko, vo = o.compact_rope(K, V, idx, base, style, pos0=pos0, offset=off)
+        new_pos = torch.tensor(pos0 + off + np.arange(len(idx)))
+        want = _rope_ref(raw[:, :, idx], new_pos.expand(nL, Hkv, len(idx)), base, style)
+        got = torch.from_numpy(ko[:, :, off:].view(np.int16)).view(torch.bfloat16).to(torch.float64)
+        err = (got - want).abs().max() / want.abs().max()
+        assert err < 2e-2, (style, float(err))
+        assert np.array_equal(vo[:, :, off:], _bits(V)[:, :, idx])
+        # positions that agree: the identity, bit for bit
+        ko0, _ = o.compact_rope(K, V, np.arange(5, 12, dtype=np.int32), base, style, pos0=5)
+        assert np.array_equal(ko0, _bits(K)[:, :, 5:12])
+
+
 def pin_gather(o):
     """Message rows (App. C.3) equal numpy fancy indexing, for hidden-state rows and token IDs."""
     rng = np.random.default_rng(4)
@@ -381,5 +422,5 @@ ALL_PINS = [
     pin_zero_denominator, pin_variance_identity, pin_identical_keys, pin_invariants,
     pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_self_keys, pin_select_golden,
     pin_select_integrity,
-    pin_compact, pin_gather,
+    pin_compact, pin_compact_rope, pin_gather,
 ]

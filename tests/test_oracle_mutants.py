@@ -59,6 +59,10 @@ MUTANTS = [
     ("self_keys_not_causal", "for (int u = 0; u <= r; ++u) Z += exp(", "for (int u = 0; u < dm->m; ++u) Z += exp("),
     ("self_keys_unscaled", "    return z * scale;\n}", "    return z;\n}"),
     ("self_keys_wrong_group", "(int64_t)g * dm->s_head;", "(int64_t)((g + 1) % dm->n_kv_heads) * dm->s_head;"),
+    ("rope_sign_flipped", "k_out[dst + a] = double_to_bf16(xa * cos(phi) - xb * sin(phi));", "k_out[dst + a] = double_to_bf16(xa * cos(phi) + xb * sin(phi));"),
+    ("rope_halves_paired_as_interleaved", "const int a = style == 0 ? k : 2 * k, b = style == 0 ? k + half : 2 * k + 1;", "const int a = 2 * k, b = 2 * k + 1;"),
+    ("rope_theta_exponent", "const double phi = delta * pow(base, -2.0 * k / d);", "const double phi = delta * pow(base, -1.0 * k / d);"),
+    ("rope_offset_dropped", "const double delta = (double)(pos0 + off + j - idx[j]);", "const double delta = (double)(pos0 + j - idx[j]);"),
     ("compact_v_from_k", "memcpy(v_out + dst, V + src, sizeof(uint16_t) * (size_t)d);", "memcpy(v_out + dst, K + src, sizeof(uint16_t) * (size_t)d);"),
 ]
 
