@@ -180,6 +180,22 @@ cb_status cb_compact(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t
                      const int64_t *out_offset, int64_t o_layer, int64_t o_head, void *stream);
 
 /*
+ * cb_compact with the positional re-index that sending K rows as they are needs (App. C.3: the
+ * paper re-prefills the selected rows at their new positions and notes that direct K/V transfer
+ * would have to handle the sender/receiver position mismatch).  Arguments as for cb_compact,
+ * plus the receiver's rotary embedding: rope_base (> 1; e.g. 1e6 for Qwen3), rope_style 0 for
+ * pairs (k, k + d/2) (rotate-half layout) or 1 for pairs (2k, 2k + 1), and pos0, the receiver
+ * position of send-buffer row 0.  Row r = out_offset[i] + j of the send buffer takes sender i's
+ * position t = idx[i][j] to receiver position pos0 + r: every pair of K's dimensions turns by
+ * (pos0 + r - t) * rope_base^(-2k/d) (rounded once to bf16); V is copied unchanged.  Errors as
+ * cb_compact, plus CB_EINVAL for a bad rope_base or rope_style.
+ */
+cb_status cb_compact_rope(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t *const *idx,
+                          const int64_t *budget, void *k_out, void *v_out, int64_t out_capacity,
+                          const int64_t *out_offset, int64_t o_layer, int64_t o_head, double rope_base,
+                          int32_t rope_style, int64_t pos0, void *stream);
+
+/*
  * Message rows by index (Sec. 3.1 "State Representation", App. C.3 "Message encoding").  The
  * continuous-row encoding sends one row of the sender's per-position table (its hidden states:
  * 8 KiB per position for Qwen3-8B) for every selected position; the token-ID encoding sends the

@@ -62,8 +62,14 @@ class Filter:
     def select(self, stream=None):
         self.cb.select(self.scores, self.Ts, self.budgets, self.idx, stream)
 
-    def compact(self, stream=None):
-        self.cb.compact(self.Ks, self.Vs, self.idx, self.budgets, self.k_out, self.v_out, self.offsets, stream)
+    def compact(self, stream=None, rope: Optional[dict] = None):
+        """rope = dict(base=..., style=0 or 1, pos0=...): also move K to receiver positions
+        pos0 + (row of the send buffer) with the receiver's rotary embedding."""
+        if rope is None:
+            self.cb.compact(self.Ks, self.Vs, self.idx, self.budgets, self.k_out, self.v_out, self.offsets, stream)
+        else:
+            self.cb.compact_rope(self.Ks, self.Vs, self.idx, self.budgets, self.k_out, self.v_out, self.offsets,
+                                 rope["base"], rope.get("style", 0), rope.get("pos0", 0), stream)
 
     def run(self, stream=None, wave: Optional[int] = None):
         """The whole path.  wave = None: score, select and compact every sender in turn on

@@ -21,7 +21,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
             "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
-            "cb_gather", "cb_chain_budget",
+            "cb_gather", "cb_chain_budget", "cb_compact_rope",
             "cb_enable_stage_timing", "cb_stage_times"]
 
 
@@ -81,6 +81,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_compact.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), P, P, P, P, ctypes.c_int64, P,
                                ctypes.c_int64, ctypes.c_int64, P]
     lib.cb_compact.restype = ctypes.c_int
+    lib.cb_compact_rope.argtypes = [P, ctypes.c_int32, ctypes.POINTER(cb_kv), P, P, P, P, ctypes.c_int64, P,
+                                    ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.c_int32,
+                                    ctypes.c_int64, P]
+    lib.cb_compact_rope.restype = ctypes.c_int
     lib.cb_gather.argtypes = [P, ctypes.c_int32, P, P, ctypes.c_int64, ctypes.c_int64, P, P, P, ctypes.c_int64, P,
                               ctypes.c_int64, P]
     lib.cb_gather.restype = ctypes.c_int
@@ -243,6 +247,20 @@ class CacheBack:
         self._check(self.lib.cb_compact(self.h, n, kv, ip, Ba, k_out.data_ptr(), v_out.data_ptr(),
                                         k_out.shape[2], Oa, k_out.stride(0), k_out.stride(1),
                                         _stream_handle(stream)))
+
+    def compact_rope(self, Ks: Sequence, Vs: Sequence, idx: Sequence, budgets: Sequence[int], k_out, v_out,
+                     offsets: Sequence[int], base: float, style: int = 0, pos0: int = 0, stream=None):
+        """compact with K moved to receiver positions pos0 + offset + j by the rotary embedding
+        (style 0: pairs (k, k + d/2); 1: pairs (2k, 2k + 1))."""
+        n = len(Ks)
+        kv = (cb_kv * n)(*[kv_desc(K, V) for K, V in zip(Ks, Vs)])
+        ip = _ptr_array([x.data_ptr() for x in idx])
+        Ba = _ptr_array([int(b) for b in budgets], ctypes.c_int64)
+        Oa = _ptr_array([int(o) for o in offsets], ctypes.c_int64)
+        assert k_out.stride(3) == 1 and k_out.stride(2) == k_out.shape[3] and v_out.stride() == k_out.stride()
+        self._check(self.lib.cb_compact_rope(self.h, n, kv, ip, Ba, k_out.data_ptr(), v_out.data_ptr(),
+                                             k_out.shape[2], Oa, k_out.stride(0), k_out.stride(1), float(base),
+                                             int(style), int(pos0), _stream_handle(stream)))
 
     def gather(self, tables: Sequence, idx: Sequence, counts: Sequence[int], out, offsets: Sequence[int],
                stream=None):

@@ -409,9 +409,22 @@ cb_status cb_select(cb_ctx* ctx, int32_t n, const float* const* scores, const in
     return CB_OK;
 }
 
-cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx, const int64_t* budget,
-                     void* k_out, void* v_out, int64_t out_capacity, const int64_t* out_offset, int64_t o_layer,
-                     int64_t o_head, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Rotary re-index of cb_compact_rope (null for cb_compact).
+struct RopeArgs {
+    double base;
+    int32_t style;
+    int64_t pos0;
+};
+
+// Shared body of cb_compact and cb_compact_rope: validation, batching, launch.
+cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx,
+                       const int64_t* budget, void* k_out, void* v_out, int64_t out_capacity,
+                       const int64_t* out_offset, int64_t o_layer, int64_t o_head, const RopeArgs* rope,
+                       void* stream) {
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     ctx->last_error.clear();
     const cb_config& c = ctx->cfg;
@@ -421,6 +434,8 @@ cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t
     if (!stride_ok(o_head) || !stride_ok(o_layer) || o_head < out_capacity * c.head_dim ||
         o_layer < (int64_t)c.n_kv_heads * o_head)
         return fail(ctx, CB_EINVAL, "output strides must be multiples of 8 and not overlap rows");
+    if (rope && (!(rope->base > 1.0) || !std::isfinite(rope->base) || (rope->style != 0 && rope->style != 1)))
+        return fail(ctx, CB_EINVAL, "rope_base must be finite and > 1, rope_style 0 or 1");
     DeviceGuard dg(ctx->device);
     if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
     cb_status st;
@@ -469,10 +484,31 @@ cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t
             d.B = budget[b0 + k];
             d.out_off = out_offset[b0 + k];
         }
-        cudaError_t e = cbk::launch_compact(bt, strm, ctx->num_sms);
+        cudaError_t e = rope ? cbk::launch_compact_rope(bt, rope->base, rope->style, rope->pos0, strm, ctx->num_sms)
+                             : cbk::launch_compact(bt, strm, ctx->num_sms);
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "compact launch failed: %s", cudaGetErrorString(e));
     }
     return CB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx, const int64_t* budget,
+                     void* k_out, void* v_out, int64_t out_capacity, const int64_t* out_offset, int64_t o_layer,
+                     int64_t o_head, void* stream) {
+    return compact_impl(ctx, n, senders, idx, budget, k_out, v_out, out_capacity, out_offset, o_layer, o_head,
+                        nullptr, stream);
+}
+
+cb_status cb_compact_rope(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx,
+                          const int64_t* budget, void* k_out, void* v_out, int64_t out_capacity,
+                          const int64_t* out_offset, int64_t o_layer, int64_t o_head, double rope_base,
+                          int32_t rope_style, int64_t pos0, void* stream) {
+    const RopeArgs r{rope_base, rope_style, pos0};
+    return compact_impl(ctx, n, senders, idx, budget, k_out, v_out, out_capacity, out_offset, o_layer, o_head, &r,
+                        stream);
 }
 
 cb_status cb_enable_stage_timing(cb_ctx* ctx, int32_t enable) {

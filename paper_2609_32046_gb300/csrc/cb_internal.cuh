@@ -152,5 +152,8 @@ cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms, int*
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);
 cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms);
 cudaError_t launch_gather(const GatherBatch& b, cudaStream_t st, int num_sms);
+// cb_compact with K rotated from sender position idx[j] to receiver position pos0 + out_off + j.
+cudaError_t launch_compact_rope(const CompactBatch& b, double base, int style, int64_t pos0, cudaStream_t st,
+                                int num_sms);
 
 }  // namespace cbk
