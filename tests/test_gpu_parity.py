@@ -36,6 +36,10 @@ CASES = [
     ("pool3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=3)),
     ("pool5_p3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=5, p=3.0)),
     ("tail_1_position", (1, 8, 2, 128), [123], 8, 0.5, {}),
+    # degenerate sizes: a single position, fewer positions than the forced 41, exactly 41
+    ("degenerate_T", (2, 8, 2, 128), [1, 2, 40, 41, 129], 3, 0.5, {}),
+    ("keep_everything", (1, 8, 2, 128), [300, 77], 5, 1.0, {}),
+    ("keep_forced_only", (1, 8, 2, 64), [500], 4, 0.01, {}),
     # p = infinity (App. D.2): maxima instead of sums of powers
     ("p_inf_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(p=float("inf"))),
     ("p_inf_g2_pool5", (2, 8, 4, 128), [611], 20, 0.3, dict(p=float("inf"), pool_width=5, alpha=3.0)),
