@@ -60,7 +60,8 @@ def workload_bytes_flops(spec, keep):
         row = sh.head_dim * 2
         kbytes = sh.n_layers * sh.n_kv_heads * T * row
         cbytes = 2 * 2 * sh.n_layers * sh.n_kv_heads * B * row   # read + write, K and V
-        score_b += kbytes
+        if not (spec.shared_sender and i > 0):       # one sender state read once for all its queries
+            score_b += kbytes
         compact_b += cbytes
         tot_f += 2 * 2 * spec.m * sh.n_q_heads * T * sh.head_dim * sh.n_layers
     tot_b = score_b + compact_b
@@ -243,8 +244,32 @@ def max_over_ranks(ws, x: float) -> float:
 # CPU oracle timing (the cpu_baseline object and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(spec_name: str, n_layers_sample: int, seed: int = 0):
-    """Time the oracle on sender 0 of the workload, scoring n_layers_sample of its layers.
+def sample_layers(spec) -> int:
+    """Layers of sender 0 the oracle scores per sample: all 36 for a Qwen3-8B-shaped sender of
+    8192 positions and 64 query tokens (a few seconds on the host cores), proportionally fewer
+    for larger T * m, so that one sample stays within seconds on every workload."""
+    work = spec.T[0] * spec.m
+    return max(1, min(spec.shape.n_layers, (36 * 8192 * 64) // work))
+
+
+_ORACLE_INPUTS = {}
+
+
+def _oracle_inputs(spec_name: str, seed: int):
+    """Sender 0 and its query on the host, generated once per process (the timed region holds
+    the oracle's work only)."""
+    key = (spec_name, seed)
+    if key not in _ORACLE_INPUTS:
+        import synth
+        spec = synth.SPECS[spec_name]
+        Q = synth.make_query(spec, seed, 0, "cpu")
+        _ORACLE_INPUTS[key] = (synth.make_sender(spec, seed, 0, Q, "cpu"), Q)
+    return _ORACLE_INPUTS[key]
+
+
+def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
+    """Time the oracle on sender 0 of the workload, scoring n_layers_sample of its layers
+    (0: sample_layers(spec)).
 
     Scoring is linear in the scored layers, so the full-workload time is the sample's
     score time x (layers / sampled layers) x senders, plus select and compact times x senders.
@@ -252,9 +277,10 @@ def oracle_sample(spec_name: str, n_layers_sample: int, seed: int = 0):
     import oracle
     import synth
     spec = synth.SPECS[spec_name]
+    if n_layers_sample <= 0:
+        n_layers_sample = sample_layers(spec)
     o = oracle.default()
-    snd = synth.make_sender(spec, seed, 0, synth.make_query(spec, seed, 0, "cpu"), "cpu")
-    Q = synth.make_query(spec, seed, 0, "cpu")
+    snd, Q = _oracle_inputs(spec_name, seed)
     nl = min(n_layers_sample, spec.shape.n_layers)
     keep = spec.keeps[len(spec.keeps) // 2] if len(spec.keeps) > 1 else spec.keeps[0]
     t0 = time.perf_counter()
@@ -289,7 +315,7 @@ def run_reference(args):
     oracle.build()
     vals = []
     for k in range(args.warmup + args.steps):
-        r = oracle_sample(args.workload, 1)
+        r = oracle_sample(args.workload)
         if k >= args.warmup:
             vals.append(r)
     v = statistics.median([x["value"] for x in vals])
@@ -326,6 +352,8 @@ def run_ours(args):
     w = synth.make_workload(args.workload, seed=rank, device=dev)
     senders = [(s.K, s.V) for s in w.senders]
     queries = [w.queries[s.task] for s in w.senders]
+    # distinct sender states (multi-query serving repeats one state across its queries)
+    states = list({K.data_ptr(): (K, V) for K, V in senders}.values())
     c = cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads, spec.shape.head_dim,
                      spec.m, max(spec.T), len(senders))
     f = cb.Filter(c, senders, queries, keep, device=dev)
@@ -413,8 +441,8 @@ def run_ours(args):
     # e2e: the same step through the C-ABI with the inputs in pinned host memory
     e2e = None
     if not args.no_e2e:
-        hK = [K.cpu().pin_memory() for K, _ in senders]
-        hV = [V.cpu().pin_memory() for _, V in senders]
+        hK = [K.cpu().pin_memory() for K, _ in states]
+        hV = [V.cpu().pin_memory() for _, V in states]
         hQ = [q.cpu().pin_memory() for q in w.queries]
         hko = torch.empty(f.k_out.shape, dtype=f.k_out.dtype).pin_memory()
         hvo = torch.empty_like(hko).pin_memory()
@@ -423,7 +451,7 @@ def run_ours(args):
         d2h = hko.numel() * 2 * 2 + sum(x.numel() * 4 for x in hidx)
 
         def e2e_step():
-            for (K, V), hk, hv in zip(senders, hK, hV):
+            for (K, V), hk, hv in zip(states, hK, hV):
                 K.copy_(hk, non_blocking=True)
                 V.copy_(hv, non_blocking=True)
             for q, hq in zip(w.queries, hQ):
@@ -460,7 +488,8 @@ def run_ours(args):
                    "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
                    "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": keep,
                    "l2": "inputs larger than L2 (K+V %.2f GB per rank), no flush" % (
-                       sum(K.numel() * 4 for K, _ in senders) / 1e9),
+                       sum(K.numel() * 4 for K, _ in states) / 1e9),
+                   "sender_states": len(states),
                    "parallelism": "replicas" if ws > 1 else "single",
                    "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential"},
         "hbm_gbs": tot_b / step_s / 1e9,
@@ -520,7 +549,7 @@ def main():
     ap.add_argument("--keep", type=float, default=None)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-layers", type=int, default=4)
+    ap.add_argument("--cpu-layers", type=int, default=0, help="oracle layers per sample (0: by workload size)")
     ap.add_argument("--wave", type=int, default=None,
                     help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()

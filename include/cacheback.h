@@ -129,6 +129,10 @@ cb_status cb_create(const cb_config *cfg, cb_ctx **out);
  * a = softmax over the sender's T positions of softmax_scale * <q_{l,r,h}, k_{l,h/G,t}>,
  * b_{s,r,t} = mean of a over the G query heads of KV group s = (l, g); C = 1 where the
  * denominator is 0 (or below FLT_MIN in fp32).  Sender i is scored against queries[i].
+ * Entries may repeat one sender cache with different queries: one launch then scores one
+ * sender state against many receiver queries (multi-query serving: Sec. 5, Discussion, notes that one
+ * completed sender state can be scored for several receiver queries), each pair exactly as if
+ * it were scored alone.
  *   n         1..max_senders;  senders, queries, scores: host arrays of n entries
  *   scores[i] device float[T_i], written; 16-byte aligned
  * Errors: CB_EINVAL (null/misaligned pointers, strides), CB_ESHAPE (T_i or m_i above the limits).

@@ -23,7 +23,9 @@ __all__ = ["CacheBack", "CBError", "budget", "chain_budget", "load_library", "LI
 class Filter:
     """Score -> select -> compact for a fixed batch of senders, outputs allocated once.
 
-    senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors
+    senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors; one (K, V) may appear several
+             times, each with its own query (multi-query serving: one launch scores the state
+             for every receiver query, and each query gets its own message)
     queries: list of Q bf16 [nL][m_i][Hq][d] device tensors, one per sender (may repeat)
     keep:    keep ratio; budgets B_i = max(ceil(keep * T_i), min(T_i, n_sink + n_latent))
     The send buffer holds every sender's rows back to back: sender i at offset sum_{j<i} B_j.

@@ -148,6 +148,7 @@ class WorkloadSpec:
     zipf_s: float = 1.1
     n_latent: int = 40
     span_width: int = 16
+    shared_sender: bool = False   # every (sender, query) pair holds sender state 0 (multi-query serving)
 
     @property
     def n_senders(self) -> int:
@@ -172,6 +173,10 @@ SPECS = {
     # concurrency sweep: 16 tasks x 3 senders x 8192, per-task query of 64 tokens
     "sweep": WorkloadSpec("sweep", QWEN3_8B, (8192,) * 3, 64, (0.10, 0.25, 0.50), 3, 16,
                           "spans", planted_frac=0.05, beta=0.5),
+    # multi-query serving: one Qwen3-8B-shaped sender state (T=8192) scored against 8 receiver
+    # queries of 64 tokens in one launch, keep 25% per query
+    "multiquery": WorkloadSpec("multiquery", QWEN3_8B, (8192,), 64, (0.25,), 1, 8,
+                               "spans", planted_frac=0.05, beta=0.5, shared_sender=True),
 }
 
 
@@ -277,12 +282,23 @@ def make_sender(spec: WorkloadSpec, seed: int, index: int, Qcpu: Optional[torch.
 def make_workload(name: str, seed: int = 0, device="cpu", senders: Optional[Sequence[int]] = None) -> Workload:
     spec = SPECS[name]
     ids = list(range(spec.n_senders)) if senders is None else list(senders)
+    return _assemble(spec, seed, device, ids)
+
+
+def _assemble(spec: WorkloadSpec, seed: int, device, ids: Sequence[int]) -> Workload:
     tasks = sorted({i // spec.senders_per_task for i in ids})
     qcpu = {t: make_query(spec, seed, t, "cpu") for t in tasks}
     queries = {t: qcpu[t].to(device) for t in tasks}
     out = []
-    for i in ids:
-        out.append(make_sender(spec, seed, i, qcpu[i // spec.senders_per_task], device))
+    if spec.shared_sender:
+        # one sender state (planted toward task 0's query); pair i scores it against task i's query
+        base = make_sender(spec, seed, 0, make_query(spec, seed, 0, "cpu"), device)
+        for i in ids:
+            out.append(Sender(K=base.K, V=base.V, task=i // spec.senders_per_task,
+                              planted_spans=base.planted_spans, planted_beta=base.planted_beta))
+    else:
+        for i in ids:
+            out.append(make_sender(spec, seed, i, qcpu[i // spec.senders_per_task], device))
     # re-map task ids to positions in the returned query list
     order = {t: k for k, t in enumerate(tasks)}
     for snd in out:
@@ -301,8 +317,4 @@ def custom_workload(shape: Shape, Ts: Sequence[int], m: int, seed: int = 0, devi
 
 
 def make_workload_from_spec(spec: WorkloadSpec, seed: int = 0, device="cpu") -> Workload:
-    ids = list(range(spec.n_senders))
-    tasks = sorted({i // spec.senders_per_task for i in ids})
-    qcpu = {t: make_query(spec, seed, t, "cpu") for t in tasks}
-    out = [make_sender(spec, seed, i, qcpu[i // spec.senders_per_task], device) for i in ids]
-    return Workload(spec=spec, seed=seed, queries=[qcpu[t].to(device) for t in tasks], senders=out)
+    return _assemble(spec, seed, device, list(range(spec.n_senders)))

@@ -153,7 +153,7 @@ def test_deterministic_across_runs_and_streams():
 
 
 def test_scores_depend_on_the_query():
-    """Sec. 5.1 ablation: an unrelated query changes the selection."""
+    """Sec. 4.2 query ablation: an unrelated query changes the selection."""
     w = synth.make_workload("tiny")
     s = w.senders[0]
     other = synth.make_query(w.spec, seed=99, task=0).cuda()
