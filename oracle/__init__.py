@@ -86,6 +86,9 @@ class Oracle:
         lib.cbo_gather.argtypes = [_P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, _P, ctypes.c_int64, _P,
                                    ctypes.c_int64, ctypes.c_int64]
         lib.cbo_gather.restype = ctypes.c_int
+        i32, i64 = ctypes.c_int32, ctypes.c_int64
+        lib.cbo_unpage.argtypes = [_P, i32, i32, i32, i64, _P, i64, i64, i64, i64, i64, i64, _P]
+        lib.cbo_unpage.restype = ctypes.c_int
         lib.cbo_pool.argtypes = [_P, _P, ctypes.c_int64, ctypes.c_int32]
         lib.cbo_pool.restype = None
         lib.cbo_max_threads.restype = ctypes.c_int
@@ -232,6 +235,20 @@ class Oracle:
                                  out.ctypes.data, offset, row_bytes)
         if st != OK:
             raise RuntimeError("cbo_gather failed with status %d" % st)
+        return out
+
+    def unpage(self, pool, pages, T: int) -> np.ndarray:
+        """Paged cache layout (App. F, vLLM's block table): pool indexed [l][page][row][g][k]
+        (P = rows per page), pages[b] = the page holding positions b*P .. b*P + P - 1.  Returns the
+        contiguous cache [nL][Hkv][T][d] as bf16 bits."""
+        pl = np.ascontiguousarray(self._raw(pool))
+        nL, n_pages, P, Hkv, d = pl.shape
+        pg = np.ascontiguousarray(pages, dtype=np.int32)
+        out = np.zeros((nL, Hkv, T, d), dtype=pl.dtype)
+        st = self.lib.cbo_unpage(pl.ctypes.data, nL, Hkv, d, T, pg.ctypes.data, P, n_pages,
+                                 n_pages * P * Hkv * d, P * Hkv * d, Hkv * d, d, out.ctypes.data)
+        if st != OK:
+            raise RuntimeError("cbo_unpage failed with status %d" % st)
         return out
 
     @staticmethod

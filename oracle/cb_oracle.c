@@ -465,6 +465,32 @@ int cbo_gather(const uint8_t *src, int64_t T, int64_t src_stride, int64_t row_by
     return CBO_OK;
 }
 
+/*
+ * Paged (block-table) cache layout (App. F: the agents are served by vLLM, whose KV cache is
+ * kept in fixed-size pages named by a per-sequence block table).  Position t of the sender is
+ * row (t mod P) of page pages[floor(t / P)], the same page in every layer and KV head:
+ *   out[l][g][t][k] = pool[l * s_layer + pages[t / P] * s_page + (t mod P) * s_pos + g * s_head + k]
+ * for t < T.  The result is the contiguous [nL][Hkv][T][d] cache the other routines read.
+ * Returns CBO_EINVAL (writing nothing) when a page entry lies outside [0, n_pages).
+ */
+int cbo_unpage(const uint16_t *pool, int32_t nL, int32_t Hkv, int32_t d, int64_t T, const int32_t *pages,
+               int64_t P, int64_t n_pages, int64_t s_layer, int64_t s_page, int64_t s_pos, int64_t s_head,
+               uint16_t *out) {
+    if (!pool || !out || (T > 0 && !pages) || nL < 1 || Hkv < 1 || d < 1 || T < 0 || P < 1) return CBO_EINVAL;
+    const int64_t n_used = (T + P - 1) / P;
+    for (int64_t b = 0; b < n_used; ++b)
+        if (pages[b] < 0 || pages[b] >= n_pages) return CBO_EINVAL;
+    for (int32_t l = 0; l < nL; ++l)
+        for (int32_t g = 0; g < Hkv; ++g)
+            for (int64_t t = 0; t < T; ++t) {
+                const int64_t page = pages[t / P], row = t % P;
+                const uint16_t *src = pool + l * s_layer + page * s_page + row * s_pos + g * s_head;
+                uint16_t *dst = out + (((int64_t)l * Hkv + g) * T + t) * d;
+                for (int32_t k = 0; k < d; ++k) dst[k] = src[k];
+            }
+    return CBO_OK;
+}
+
 /* double -> bf16 bits, rounded once to nearest (ties to even); finite normal inputs. */
 static uint16_t double_to_bf16(double x) {
     if (x == 0.0) return signbit(x) ? 0x8000u : 0u;

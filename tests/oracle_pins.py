@@ -417,10 +417,37 @@ def pin_gather(o):
     assert np.array_equal(o.gather(ids, idx), ids[idx])
 
 
+def pin_unpage(o):
+    """Paged layout (App. F, vLLM block table): a hand-traced table, a single identity page,
+    and a second layer / head reading the same table; a page entry outside the pool is refused."""
+    # 1 layer, 1 KV head, d = 2, P = 2, 3 pages; element value = 100 * page + 10 * row + k
+    pool = np.array([[[[[100 * p + 10 * r + k for k in range(2)]] for r in range(2)] for p in range(3)]],
+                    dtype=np.uint16)                       # [1][3][2][1][2]
+    got = o.unpage(pool, [2, 0, 1], 5)[0, 0]
+    # positions 0..4 -> (page, row) = (2,0) (2,1) (0,0) (0,1) (1,0), traced by hand
+    want = np.array([[200, 201], [210, 211], [0, 1], [10, 11], [100, 101]], dtype=np.uint16)
+    assert np.array_equal(got, want), got
+    # one page holding every position in order: the pool itself, rearranged to [l][g][t][k]
+    rng = np.random.default_rng(6)
+    one = rng.integers(0, 1 << 16, size=(2, 1, 7, 3, 4), dtype=np.uint16)
+    assert np.array_equal(o.unpage(one, [0], 7), one[:, 0].transpose(0, 2, 1, 3))
+    # two layers, two heads: layer 1 / head 1 of position 3 comes from page 0, row 1 (P = 2, pages [1, 0])
+    big = rng.integers(0, 1 << 16, size=(2, 2, 2, 2, 4), dtype=np.uint16)
+    u = o.unpage(big, [1, 0], 4)
+    assert np.array_equal(u[1, 1, 3], big[1, 0, 1, 1]) and np.array_equal(u[0, 1, 0], big[0, 1, 0, 1])
+    assert np.array_equal(u[1, 0, 2], big[1, 0, 0, 0]) and np.array_equal(u[0, 0, 1], big[0, 1, 1, 0])
+    try:
+        o.unpage(pool, [2, 3, 1], 5)
+    except RuntimeError:
+        pass
+    else:
+        raise AssertionError("a page entry outside the pool was accepted")
+
+
 ALL_PINS = [
     pin_pool_one_hot, pin_pool_library, pin_attention_sdpa, pin_one_hot_closed_form,
     pin_zero_denominator, pin_variance_identity, pin_identical_keys, pin_invariants,
     pin_special_cases, pin_equivariance, pin_brute, pin_p_infinity, pin_self_keys, pin_select_golden,
     pin_select_integrity,
-    pin_compact, pin_compact_rope, pin_gather,
+    pin_compact, pin_compact_rope, pin_gather, pin_unpage,
 ]

@@ -58,6 +58,10 @@ MUTANTS = [
     ("gather_row_shifted", "memcpy(out + (off + j) * out_stride, src + (int64_t)idx[j] * src_stride, (size_t)row_bytes);", "memcpy(out + (off + j) * out_stride, src + (int64_t)(idx[j] + (idx[j] + 1 < T)) * src_stride, (size_t)row_bytes);"),
     ("self_keys_not_causal", "for (int u = 0; u <= r; ++u) Z += exp(", "for (int u = 0; u < dm->m; ++u) Z += exp("),
     ("self_keys_unscaled", "    return z * scale;\n}", "    return z;\n}"),
+    ("unpage_pages_in_order", "const int64_t page = pages[t / P], row", "const int64_t page = t / P, row"),
+    ("unpage_row_dropped", "page * s_page + row * s_pos + g * s_head", "page * s_page + g * s_head"),
+    ("unpage_layer_stride_dropped", "pool + l * s_layer + page * s_page", "pool + page * s_page"),
+    ("unpage_head_stride_dropped", "row * s_pos + g * s_head;", "row * s_pos;"),
     ("self_keys_wrong_group", "(int64_t)g * dm->s_head;", "(int64_t)((g + 1) % dm->n_kv_heads) * dm->s_head;"),
     ("rope_sign_flipped", "k_out[dst + a] = double_to_bf16(xa * cos(phi) - xb * sin(phi));", "k_out[dst + a] = double_to_bf16(xa * cos(phi) + xb * sin(phi));"),
     ("rope_halves_paired_as_interleaved", "const int a = style == 0 ? k : 2 * k, b = style == 0 ? k + half : 2 * k + 1;", "const int a = 2 * k, b = 2 * k + 1;"),
