@@ -341,6 +341,27 @@ def run_reference(args):
 # GPU arm
 # ---------------------------------------------------------------------------
 
+def paged_cache(cb, K, V, P: int, seed: int = 0):
+    """K, V [nL][Hkv][T][d] copied into pools of pages [nL][n_pages][P][Hkv][d] (vLLM's per-layer
+    cache layout stacked over layers) in a random page order; returns the PagedKV."""
+    import torch
+    nL, Hkv, T, d = K.shape
+    nb = (T + P - 1) // P
+    g = torch.Generator().manual_seed(seed)
+    order = torch.randperm(nb, generator=g).to(K.device)
+    pools = []
+    for X in (K, V):
+        pool = torch.zeros((nL, nb, P, Hkv, d), dtype=X.dtype, device=X.device)
+        for b0 in range(0, nb, 64):           # in slices, to bound the temporary memory
+            b1 = min(nb, b0 + 64)
+            t0, t1 = b0 * P, min(T, b1 * P)
+            blk = X.new_zeros(nL, Hkv, (b1 - b0) * P, d)
+            blk[:, :, :t1 - t0] = X[:, :, t0:t1]
+            pool[:, order[b0:b1]] = blk.view(nL, Hkv, b1 - b0, P, d).permute(0, 2, 3, 1, 4)
+        pools.append(pool)
+    return cb.PagedKV(pools[0], pools[1], order.to(torch.int32), T)
+
+
 def run_ours(args):
     import torch
     import paper_2609_32046_gb300 as cb
@@ -356,7 +377,16 @@ def run_ours(args):
     states = list({K.data_ptr(): (K, V) for K, V in senders}.values())
     c = cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads, spec.shape.head_dim,
                      spec.m, max(spec.T), len(senders))
-    f = cb.Filter(c, senders, queries, keep, device=dev)
+    if args.paged:
+        # the same caches in a vLLM-style paged layout: pages of args.paged positions in a random order
+        pk = {K.data_ptr(): paged_cache(cb, K, V, args.paged, seed=rank) for K, V in states}
+        f = cb.Filter(c, [pk[K.data_ptr()] for K, _ in senders], queries, keep, device=dev)
+        inputs = [(p.k_pool, p.v_pool) for p in pk.values()]      # what the end-to-end step uploads
+        states = None
+        torch.cuda.empty_cache()
+    else:
+        f = cb.Filter(c, senders, queries, keep, device=dev)
+        inputs = states
     stream = torch.cuda.current_stream(dev)
     n_send = len(senders)
     # --wave w: senders in waves on two streams (a wave's selection and compaction queued beside the
@@ -441,8 +471,8 @@ def run_ours(args):
     # e2e: the same step through the C-ABI with the inputs in pinned host memory
     e2e = None
     if not args.no_e2e:
-        hK = [K.cpu().pin_memory() for K, _ in states]
-        hV = [V.cpu().pin_memory() for _, V in states]
+        hK = [K.cpu().pin_memory() for K, _ in inputs]
+        hV = [V.cpu().pin_memory() for _, V in inputs]
         hQ = [q.cpu().pin_memory() for q in w.queries]
         hko = torch.empty(f.k_out.shape, dtype=f.k_out.dtype).pin_memory()
         hvo = torch.empty_like(hko).pin_memory()
@@ -451,7 +481,7 @@ def run_ours(args):
         d2h = hko.numel() * 2 * 2 + sum(x.numel() * 4 for x in hidx)
 
         def e2e_step():
-            for (K, V), hk, hv in zip(states, hK, hV):
+            for (K, V), hk, hv in zip(inputs, hK, hV):
                 K.copy_(hk, non_blocking=True)
                 V.copy_(hv, non_blocking=True)
             for q, hq in zip(w.queries, hQ):
@@ -488,8 +518,10 @@ def run_ours(args):
                    "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
                    "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": keep,
                    "l2": "inputs larger than L2 (K+V %.2f GB per rank), no flush" % (
-                       sum(K.numel() * 4 for K, _ in states) / 1e9),
-                   "sender_states": len(states),
+                       sum(K.numel() * 4 for K, _ in inputs) / 1e9),
+                   "sender_states": len(inputs),
+                   "layout": ("paged: %d positions per page, pages in a random order" % args.paged)
+                             if args.paged else "strided [nL][Hkv][T][d]",
                    "parallelism": "replicas" if ws > 1 else "single",
                    "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential"},
         "hbm_gbs": tot_b / step_s / 1e9,
@@ -550,6 +582,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-layers", type=int, default=0, help="oracle layers per sample (0: by workload size)")
+    ap.add_argument("--paged", type=int, default=0,
+                    help="hold each sender cache in pages of this many positions (random page order)")
     ap.add_argument("--wave", type=int, default=None,
                     help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()

@@ -88,11 +88,30 @@ typedef struct {
 } cb_config;
 
 /* One sender's cache M_S (App. A): K[l][g][t][:] at k + l*s_layer + g*s_head + t*s_pos,
- * V likewise with the same strides.  T = number of cached positions (T_i = H_i + G_i, Sec. 2). */
+ * V likewise with the same strides.  T = number of cached positions (T_i = H_i + G_i, Sec. 2).
+ *
+ * Paged layout (optional; App. F: the agents run under vLLM, whose cache lives in fixed-size
+ * pages named by a per-sequence block table).  With pages != NULL, position t is row
+ * t % page_size of page pages[t / page_size], the same page in every layer and KV head:
+ *   K[l][g][t][:] at k + l*s_layer + g*s_head + pages[t / page_size]*s_page + (t % page_size)*s_pos
+ * and V likewise (same table, same strides).  vLLM's per-layer [n_pages][page_size][Hkv][d]
+ * caches stacked over layers give s_layer = n_pages*page_size*Hkv*d, s_page = page_size*Hkv*d,
+ * s_pos = Hkv*d, s_head = d.
+ *   pages      device int32[ceil(T / page_size)] (4-byte aligned), read by the kernels; NULL
+ *              selects the strided layout and the three fields below are ignored
+ *   page_size  rows per page, a power of two in 1..65536
+ *   s_page     elements between consecutive pages: a positive multiple of 8
+ *   n_pages    pages in the pool; an entry outside [0, n_pages) is never dereferenced: its rows
+ *              read as zero (cb_score) or are not written (cb_compact*), and the next
+ *              cb_sync_status() reports CB_EDEVICE
+ * cb_score, cb_compact and cb_compact_rope take either layout, sender by sender. */
 typedef struct {
     const void *k, *v;
     int64_t T;
     int64_t s_layer, s_head, s_pos;
+    const int32_t *pages;
+    int32_t page_size;
+    int64_t s_page, n_pages;
 } cb_kv;
 
 /* The receiver query's post-RoPE query vectors in the sender's scored layers (Sec. 3:

@@ -14,16 +14,18 @@ from __future__ import annotations
 from typing import List, Optional, Sequence
 
 from .binding import (CB_EBUDGET, CB_ECUDA, CB_EDEVICE, CB_EINVAL, CB_ENOMEM, CB_ESHAPE, CB_OK, EXPORTED,
-                      LIB_PATH, CacheBack, CBError, budget, chain_budget, load_library)
+                      LIB_PATH, CacheBack, CBError, PagedKV, budget, chain_budget, load_library)
 
-__all__ = ["CacheBack", "CBError", "budget", "chain_budget", "load_library", "LIB_PATH", "EXPORTED", "Filter", "Chain",
+__all__ = ["CacheBack", "CBError", "PagedKV", "budget", "chain_budget", "load_library", "LIB_PATH", "EXPORTED",
+           "Filter", "Chain",
            "CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_EDEVICE"]
 
 
 class Filter:
     """Score -> select -> compact for a fixed batch of senders, outputs allocated once.
 
-    senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors; one (K, V) may appear several
+    senders: list of (K, V) bf16 [nL][Hkv][T_i][d] device tensors, or PagedKV caches (block-table
+             layout); one (K, V) may appear several
              times, each with its own query (multi-query serving: one launch scores the state
              for every receiver query, and each query gets its own message)
     queries: list of Q bf16 [nL][m_i][Hq][d] device tensors, one per sender (may repeat)
@@ -35,6 +37,8 @@ class Filter:
                  query_keys: Optional[Sequence] = None):
         import torch
         self.cb = cb
+        # a PagedKV stands for both K and V of its sender
+        senders = [(s, s) if isinstance(s, PagedKV) else s for s in senders]
         self.Ks = [k for k, _ in senders]
         self.Vs = [v for _, v in senders]
         self.Qs = list(queries)

@@ -43,7 +43,9 @@ class cb_config(ctypes.Structure):
 
 class cb_kv(ctypes.Structure):
     _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("T", ctypes.c_int64),
-                ("s_layer", ctypes.c_int64), ("s_head", ctypes.c_int64), ("s_pos", ctypes.c_int64)]
+                ("s_layer", ctypes.c_int64), ("s_head", ctypes.c_int64), ("s_pos", ctypes.c_int64),
+                ("pages", ctypes.c_void_p), ("page_size", ctypes.c_int32), ("s_page", ctypes.c_int64),
+                ("n_pages", ctypes.c_int64)]
 
 
 class cb_query(ctypes.Structure):
@@ -152,8 +154,42 @@ def _stream_handle(stream) -> int:
     return stream.cuda_stream
 
 
+class PagedKV:
+    """A sender cache in the paged (block-table) layout of a vLLM-style server (App. F).
+
+    k_pool, v_pool: bf16 tensors indexed [l][page][row][g][k] (vLLM's per-layer
+                    [n_pages][page_size][Hkv][d] caches stacked over layers, or any view with
+                    that index order and a unit head-dim stride; both with the same strides)
+    pages:          int32 device tensor, pages[b] = the page holding positions
+                    b * page_size .. b * page_size + page_size - 1 (the sequence's block table)
+    T:              positions cached
+    Quacks like the [nL][Hkv][T][d] tensor it stands for (shape, dtype, device), so it can be
+    passed wherever a sender's K is expected; kv_desc(p) describes both pools.
+    """
+
+    def __init__(self, k_pool, v_pool, pages, T: int):
+        assert k_pool.dim() == 5 and k_pool.dtype.itemsize == 2 and k_pool.stride(4) == 1
+        assert v_pool.shape == k_pool.shape and v_pool.stride() == k_pool.stride()
+        nL, n_pages, P, Hkv, d = k_pool.shape
+        assert P & (P - 1) == 0, "page_size must be a power of two"
+        assert pages.dtype.itemsize == 4 and pages.is_contiguous() and pages.numel() >= (T + P - 1) // P
+        self.k_pool, self.v_pool, self.pages, self.T = k_pool, v_pool, pages, int(T)
+        self.page_size, self.n_pages = P, n_pages
+        self.shape = (nL, Hkv, int(T), d)
+        self.dtype = k_pool.dtype
+        self.device = k_pool.device
+
+    def desc(self) -> cb_kv:
+        k = self.k_pool
+        return cb_kv(k.data_ptr(), self.v_pool.data_ptr(), self.T, k.stride(0), k.stride(3), k.stride(2),
+                     self.pages.data_ptr(), self.page_size, k.stride(1), self.n_pages)
+
+
 def kv_desc(K, V=None) -> cb_kv:
-    """K, V: bf16 [nL][Hkv][T][d] (any strides with unit head-dim stride)."""
+    """K, V: bf16 [nL][Hkv][T][d] (any strides with unit head-dim stride), or K a PagedKV
+    (V ignored: the PagedKV holds both pools)."""
+    if isinstance(K, PagedKV):
+        return K.desc()
     assert K.dtype.itemsize == 2 and K.stride(3) == 1
     if V is not None:
         assert V.shape == K.shape and V.stride() == K.stride()

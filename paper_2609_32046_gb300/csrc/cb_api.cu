@@ -119,6 +119,30 @@ cb_status check_device_ptr(cb_ctx* ctx, const void* p, const char* what, int i, 
 
 bool stride_ok(int64_t s) { return s > 0 && (s % 8) == 0; }
 
+// The optional block table of a sender (paged layout).
+cb_status check_pages(cb_ctx* ctx, const cb_kv& s, int i) {
+    if (!s.pages) return CB_OK;
+    if (s.page_size < 1 || s.page_size > 65536 || (s.page_size & (s.page_size - 1)) != 0)
+        return fail(ctx, CB_EINVAL, "senders[%d].page_size = %d is not a power of two in [1, 65536]", i,
+                    s.page_size);
+    if (!stride_ok(s.s_page)) return fail(ctx, CB_EINVAL, "senders[%d].s_page must be a positive multiple of 8", i);
+    if (s.n_pages < 1) return fail(ctx, CB_EINVAL, "senders[%d].n_pages must be at least 1", i);
+    return check_device_ptr(ctx, s.pages, "senders.pages", i, 4);
+}
+
+cbk::PageMap page_map(const cb_kv& s) {
+    cbk::PageMap pm{};
+    if (s.pages) {
+        pm.pages = s.pages;
+        pm.s_page = s.s_page;
+        pm.n_pages = s.n_pages;
+        int sh = 0;
+        while ((1 << sh) < s.page_size) ++sh;
+        pm.shift = sh;
+    }
+    return pm;
+}
+
 template <typename T>
 cudaError_t alloc(T** p, size_t count, int64_t* total) {
     if (count == 0) count = 1;
@@ -296,6 +320,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             return fail(ctx, CB_EINVAL, "queries[%d]: strides must be positive multiples of 8 (s_head >= d)", i);
         cb_status st;
         if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
+        if ((st = check_pages(ctx, s, i))) return st;
         if ((st = check_device_ptr(ctx, q.q, "queries.q", i))) return st;
         if (q.k_self) {
             if (!stride_ok(q.ks_layer) || !stride_ok(q.ks_tok) || !stride_ok(q.ks_head) || q.ks_head < c.head_dim)
@@ -339,6 +364,7 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.scores = scores[b0 + k];
             d.T = s.T;
             d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
+            d.pm = page_map(s);
             d.qs_l = q.s_layer; d.qs_t = q.s_tok; d.qs_h = q.s_head;
             d.kself = static_cast<const uint16_t*>(q.k_self);
             d.kss_l = q.ks_layer; d.kss_t = q.ks_tok; d.kss_h = q.ks_head;
@@ -457,6 +483,7 @@ cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32
             return fail(ctx, CB_EINVAL, "senders[%d]: strides must be positive multiples of 8 (s_pos >= d)", i);
         if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
         if ((st = check_device_ptr(ctx, s.v, "senders.v", i))) return st;
+        if ((st = check_pages(ctx, s, i))) return st;
         if (budget[i] > 0 && (st = check_device_ptr(ctx, idx[i], "idx", i))) return st;
     }
     cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
@@ -481,6 +508,7 @@ cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32
             d.idx = idx[b0 + k];
             d.T = s.T;
             d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
+            d.pm = page_map(s);
             d.B = budget[b0 + k];
             d.out_off = out_offset[b0 + k];
         }
@@ -618,10 +646,11 @@ cb_status cb_sync_status(cb_ctx* ctx, void* stream) {
             return fail(ctx, CB_ETIMEOUT,
                         "a bounded device wait gave up (code 0x%x: bits 8+ name the wait); the results are invalid",
                         word);
-        return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s%s)", word,
+        return fail(ctx, CB_EDEVICE, "kernel bounds check failed (code 0x%x:%s%s%s%s)", word,
                     (word & cbk::kErrCompactIndex) ? " compact index outside [0, T)" : "",
                     (word & cbk::kErrSelectBudget) ? " select count mismatch" : "",
-                    (word & cbk::kErrGatherIndex) ? " gather index outside [0, T)" : "");
+                    (word & cbk::kErrGatherIndex) ? " gather index outside [0, T)" : "",
+                    (word & cbk::kErrPageIndex) ? " block-table entry outside [0, n_pages)" : "");
     }
     return CB_OK;
 }

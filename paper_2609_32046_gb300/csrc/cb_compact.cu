@@ -5,8 +5,9 @@
 // consecutive threads copy consecutive 16-byte pieces of consecutive output rows
 // (coalesced stores, one index load per row, no per-piece division).  Each thread moves UNROLL pieces
 // per iteration with all loads issued before the stores, keeping enough bytes in
-// flight for HBM; loads bypass L1 and stores are marked streaming.  Indices are
-// bounds-checked: a bad one is skipped and recorded in the device error word.
+// flight for HBM; loads bypass L1 and stores are marked streaming.  Indices (and, for a paged
+// cache, block-table entries) are bounds-checked: a bad one is skipped and recorded in the
+// device error word.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -61,7 +62,12 @@ __global__ void __launch_bounds__(kThreads) k_compact(const __grid_constant__ Co
                 atomicOr(bt.err, kErrCompactIndex);
                 continue;
             }
-            val[u] = ld_stream(reinterpret_cast<const uint4*>(src + (int64_t)t * sd.ks_p + ch * 8));
+            const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
+            if (ro < 0) {
+                atomicOr(bt.err, kErrPageIndex);
+                continue;
+            }
+            val[u] = ld_stream(reinterpret_cast<const uint4*>(src + ro + ch * 8));
             ok[u] = true;
         }
 #pragma unroll

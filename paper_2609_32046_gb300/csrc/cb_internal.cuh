@@ -29,6 +29,25 @@ constexpr uint32_t kErrCompactIndex = 1u;
 constexpr uint32_t kErrSelectBudget = 2u;
 constexpr uint32_t kErrTimeout = 4u;       // a bounded mbarrier wait gave up
 constexpr uint32_t kErrGatherIndex = 8u;   // a message-row index outside [0, T)
+constexpr uint32_t kErrPageIndex = 16u;    // a block-table entry outside [0, n_pages)
+
+// Paged cache layout (block table): position t is row t & (2^shift - 1) of page
+// pages[t >> shift].  pages == nullptr: the strided layout, position t at t * s_pos.
+struct PageMap {
+    const int32_t* pages;
+    int64_t s_page;
+    int64_t n_pages;
+    int32_t shift;            // log2(page_size)
+};
+
+// Elements from the (l, g) base of a sender's cache to position t's row, or -1 when the
+// block-table entry lies outside [0, n_pages) (the row must not be read).
+__device__ __forceinline__ int64_t row_offset(const PageMap& pm, int64_t s_pos, int64_t t) {
+    if (!pm.pages) return t * s_pos;
+    const int32_t page = __ldg(pm.pages + (t >> pm.shift));
+    if (page < 0 || page >= pm.n_pages) return -1;
+    return (int64_t)page * pm.s_page + (t & ((int64_t(1) << pm.shift) - 1)) * s_pos;
+}
 
 // Optional per-kernel timing of the score step (owned by the context; see cb_stage_times).
 struct StageTimer;
@@ -42,6 +61,7 @@ struct ScoreSender {
     float* scores;            // [T]
     int64_t T;
     int64_t ks_l, ks_h, ks_p;
+    PageMap pm;               // paged layout of K, or pages == nullptr
     int64_t qs_l, qs_t, qs_h;
     const uint16_t* kself;    // the query tokens' own keys Ks[l][u][g][:] or null
     int64_t kss_l, kss_t, kss_h;
@@ -104,6 +124,7 @@ struct CompactSender {
     const int32_t* idx;
     int64_t T;
     int64_t ks_l, ks_h, ks_p;
+    PageMap pm;               // paged layout of K and V, or pages == nullptr
     int64_t B;
     int64_t out_off;
     int64_t row_begin;        // first row (of n_layers*n_kv_heads*B*2) of this sender

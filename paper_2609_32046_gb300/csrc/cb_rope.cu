@@ -80,7 +80,12 @@ __global__ void __launch_bounds__(kThreads) k_compact_rope(const __grid_constant
             atomicOr(bt.err, kErrCompactIndex);
             continue;
         }
-        const uint16_t* srow = src + (int64_t)t * sd.ks_p;
+        const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
+        if (ro < 0) {
+            atomicOr(bt.err, kErrPageIndex);
+            continue;
+        }
+        const uint16_t* srow = src + ro;
         uint16_t* drow = dst + j * D;
         if (kv) {
             st_stream(reinterpret_cast<uint4*>(drow + ch * 8), ld_stream(reinterpret_cast<const uint4*>(srow + ch * 8)));

@@ -81,19 +81,23 @@ __device__ __forceinline__ int find_sender(int n, int64_t blk, F begin_of) {
 
 // Stage K rows [tbase, tbase + npos) of one (l, g) slice into smem as 16-byte
 // chunks, chunk c of row n stored at column c ^ (n & 7) (conflict-free ldmatrix).
-// Rows outside [0, T) are zero.
+// Rows outside [0, T), and rows whose block-table entry is out of range (recorded in the
+// error word), are zero.
 template <int D>
-__device__ __forceinline__ void stage_keys(uint4* ksm, const uint16_t* kbase, int64_t ks_p, int64_t tbase,
-                                           int npos, int64_t T) {
+__device__ __forceinline__ void stage_keys(uint4* ksm, const uint16_t* kbase, int64_t ks_p, const PageMap& pm,
+                                           int64_t tbase, int npos, int64_t T, uint32_t* err) {
     constexpr int CH = D / 8;
     for (int e = threadIdx.x; e < npos * CH; e += kThreads) {
         const int n = e / CH, ch = e % CH;
         uint4* dst = ksm + n * CH + (ch ^ (n & 7));
         const int64_t t = tbase + n;
-        if (t >= 0 && t < T)
-            cp_async16(dst, kbase + t * ks_p + ch * 8);
-        else
+        const int64_t ro = (t >= 0 && t < T) ? row_offset(pm, ks_p, t) : -1;
+        if (ro >= 0) {
+            cp_async16(dst, kbase + ro + ch * 8);
+        } else {
             *dst = make_uint4(0u, 0u, 0u, 0u);
+            if (t >= 0 && t < T && ch == 0) atomicOr(err, kErrPageIndex);
+        }
     }
     cp_async_wait_all();
     __syncthreads();
@@ -171,7 +175,8 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
     const int s = (int)(local / sd.n_chunk1), c = (int)(local % sd.n_chunk1);
     const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
     const int64_t T = sd.T, t0 = (int64_t)c * kStatsChunk;
-    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, t0, kStatsChunk, T);
+    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, sd.pm, t0, kStatsChunk, T,
+                  bt.err);
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int qd = lane & 3, rr = lane >> 2;
@@ -377,7 +382,8 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
     const int R = sd.m * G;
     for (int row = threadIdx.x; row < R; row += kThreads) offs[row] = bt.offs[sd.offs_off + (int64_t)s * R + row];
     for (int k = threadIdx.x; k < kAccumPos; k += kThreads) bsum[k] = 0.f;
-    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, tbase, kAccumPos, T);
+    stage_keys<D>(ksm, sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h, sd.ks_p, sd.pm, tbase, kAccumPos, T,
+                  bt.err);
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int qd = lane & 3, rr = lane >> 2;

@@ -2,27 +2,27 @@
 //
 // Both passes contract the receiver query Q_s = [(r, h) rows x d] of one KV group
 // s = (l, g) with that group's keys K_s = [positions x d] (App. C.1: a_{l,h,r,t} is the
-// softmax over t of scale * <q, k>).  Operands are K-major bf16 tiles staged by TMA
-// with the 128-byte swizzle; one thread issues tcgen05.mma (fp32 accumulation in
-// TMEM); eight epilogue warps read TMEM with tcgen05.ld.
+// softmax over t of scale * <q, k>).  Operands are K-major bf16 tiles in the 128-byte
+// swizzled layout, staged by TMA (or, for a paged cache, by the producer warp's cp.async);
+// one thread issues tcgen05.mma (fp32 accumulation in TMEM); the epilogue warps read TMEM
+// with tcgen05.ld.
 //
 //   k_stats_tc  pass 1, D = Q_s K_tile^T: TMEM lane = row (r, h), column = position.
 //               Each epilogue thread owns one row and keeps its running max and
-//               sum of exp2 over the positions of a 512-position chunk.
-//   k_accum_tc  pass 2, D = K_tile Q_s^T: TMEM lane = position, column = row (r, h).
-//               Each thread owns one position: exp2(z - offset) (offset = row max +
-//               log2 of the row sum + log2 G, so the value is a / G), the head mean b
-//               and the sum over tokens stay in registers; Pool over positions runs
-//               across lanes with shuffles plus a shared-memory halo between warps.
-//               A tile is 128 positions starting 3 before its 122 output positions.
+//               sum of exp2 over its group's tiles of a 1024-position chunk.
+//   k_accum_tc  pass 2, D = K_tile Q_s^T (+ a ninth K-step of ones x the rows' offset terms,
+//               so TMEM holds z - offset / scale): TMEM lane = position, column = row (r, h).
+//               Each thread owns one position: exp2 of its logits (a / G), the head mean b
+//               and the sums over tokens stay in registers; Pool over positions runs
+//               across lanes with shuffles.  A tile's four 32-row quarters start 3 positions
+//               before their 26 output positions (104 per tile).
 //
-// Warp roles (320 threads, one CTA per SM, persistent over a contiguous range of
-// work units): warp 0 TMA producer, warp 1 MMA issuer and TMEM owner, warps 2-9
-// epilogue (two groups of four; warp w reads TMEM lanes 32*(w%4)..+31, the two
-// groups split the columns).  K tiles flow through a ring of smem stages; TMEM
-// holds two 256-column accumulator buffers.  Every mbarrier wait is bounded (1 s);
-// on a timeout the kernel records kErrTimeout, drains its copies and MMAs, frees
-// TMEM and returns.
+// Warp roles (576 threads, one CTA per SM, persistent over a contiguous range of work
+// units): warp 0 producer, warp 1 MMA issuer and TMEM owner, warps 2-17 epilogue (two
+// groups of eight taking alternate tiles; warp w reads TMEM lanes 32*(w%4)..+31).  K tiles
+// flow through a ring of smem stages; TMEM holds four 128-column accumulator buffers.
+// Every mbarrier wait is bounded (1 s); on a timeout the kernel records kErrTimeout, drains
+// its copies and MMAs, frees TMEM and returns.
 #include <cfloat>
 #include <cstdint>
 #include <cuda.h>
@@ -67,6 +67,10 @@ struct TcSender {
     int32_t ebox_rows, n_ebox;
     float inv_m, inv_mh;  // 1 / m and 1 / (m Hkv)
     int64_t unit1_begin, unit2_begin;
+    // paged cache (batches with paged != 0): K rows are copied by the producer warp
+    const uint16_t* k;
+    int64_t ks_l, ks_h, ks_p;
+    PageMap pm;
 };
 
 struct TcBatch {
@@ -76,10 +80,12 @@ struct TcBatch {
     int32_t stages, rpad_max;
     float sl2e, p;
     int32_t p_is_2, p_inf, ph;
+    int32_t paged;        // every sender of the batch has a block table (else none has)
     int64_t units1, units2;
     uint32_t* err;
     TcSender s[kMaxTcSenders];
 };
+static_assert(sizeof(TcBatch) <= 32000, "kernel parameter space");
 
 struct Ctl {
     uint64_t k_full[kMaxStages], k_empty[kMaxStages];
@@ -241,6 +247,70 @@ __device__ __forceinline__ void load_k(const TcSender& sd, const Smem& sm, int s
     tma_load_4d(dst + kTileBytes / 2, &sd.kmap, &sm.ctl->k_full[stage], 64, t_start, g, l);
 }
 
+// ---------------------------------------------------------------------------
+// Paged cache: the producer warp copies K tiles with cp.async.  Row r of a tile holds position
+// pos(r) (zero outside [0, T) and for a block-table entry outside the pool, which is recorded
+// in the error word), in the layout the TMA path writes: 64-column block kb at kb * 16 KB,
+// row r at r * 128 B, 16-byte piece j at (j ^ (r & 7)) * 16 (the 128-byte swizzle).
+// Completion runs through cp.async groups, one per tile: after committing tile k the warp
+// waits until `lag` groups at most are in flight, so tile k - lag has landed; each lane then
+// fences its writes into the async proxy that tcgen05.mma reads through, and lane 0 arrives
+// on the tile's k_full barrier (count 1, no transaction bytes).  Tiles held back this way
+// must all be published before the producer waits for the MMA issuer (q_empty), which
+// releases Q only after consuming every tile of the previous group.
+// ---------------------------------------------------------------------------
+template <typename Pos>
+__device__ __forceinline__ void copy_tile_paged(const TcSender& sd, uint8_t* dst, int l, int g, Pos pos, int lane,
+                                                uint32_t* err) {
+    const uint16_t* base = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
+    int64_t ro[4];   // element offsets of rows lane, lane + 32, lane + 64, lane + 96 (-1: zero row)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int64_t t = pos(q * 32 + lane);
+        ro[q] = -1;
+        if (t >= 0 && t < sd.T) {
+            ro[q] = row_offset(sd.pm, sd.ks_p, t);
+            if (ro[q] < 0) atomicOr(err, kErrPageIndex);
+        }
+    }
+    // lanes 0-15 copy the 16 pieces of row 2i, lanes 16-31 those of row 2i + 1
+    const int hr = lane >> 4, piece = lane & 15, kb = piece >> 3, j = piece & 7;
+    const uint32_t d0 = smem_u32(dst) + (uint32_t)kb * (kTileBytes / 2);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+#pragma unroll 4
+        for (int i = 0; i < 16; ++i) {
+            const int r = q * 32 + 2 * i + hr;
+            const int64_t o = __shfl_sync(0xffffffffu, ro[q], 2 * i + hr);
+            const uint32_t d = d0 + (uint32_t)r * 128u + ((uint32_t)(j ^ (r & 7)) << 4);
+            if (o >= 0)
+                cp_async16_zfill(d, base + o + kb * 64 + j * 8, 16u);
+            else
+                cp_async16_zfill(d, base, 0u);
+        }
+    }
+    cp_async_commit();
+}
+
+// Publish tiles [pub, kt - keep): wait until at most `keep` (0, 1 or 2) of this thread's groups
+// are in flight, fence, and arrive on their k_full barriers.  The producer keeps `lag` tiles in
+// flight in steady state and publishes everything (keep = 0) before it waits on anything the
+// MMA issuer releases only after consuming those tiles (q_empty), and at the end.
+__device__ __forceinline__ void paged_publish(Ctl* ctl, int stages, int64_t& pub, int64_t kt, int keep, int lane) {
+    if (kt - pub <= keep) return;
+    if (keep >= 2)
+        cp_async_wait<2>();
+    else if (keep == 1)
+        cp_async_wait<1>();
+    else
+        cp_async_wait<0>();
+    fence_proxy_async();
+    __syncwarp();
+    if (lane == 0)
+        for (int64_t k = pub; k < kt - keep; ++k) mbar_arrive(&ctl->k_full[k % stages]);
+    pub = kt - keep;
+}
+
 // One K = 128 contraction (8 UMMA K-steps).  a_base / b_base: first column block of each
 // operand (rows of 128 B); the second column block sits `a_blk` / `b_blk` bytes later.
 // The descriptors are built once; a K-step only moves the start-address field.
@@ -318,7 +388,44 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     my_range(bt.units1, &ub, &ue);
     const int stages = bt.stages;
 
-    if (warp == 0) {
+    if (warp == 0 && bt.paged) {
+        // ---------------- producer, paged cache: K rows by cp.async (whole warp) ----------------
+        const int lag = stages / 2;
+        int64_t kt = 0, pub = 0, qn = 0;   // tiles issued, tiles published, Q loads issued
+        int st = 0;
+        uint32_t ph = 0;
+        int prev = -1;
+        bool ok = true;
+        Unit un = decode1(bt, ub);
+        for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
+            const TcSender& sd = bt.s[un.i];
+            const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
+            const int key = un.i * 65536 + un.s;
+            if (key != prev) {
+                paged_publish(ctl, stages, pub, kt, 0, lane);   // q_empty needs the MMA past these
+                if (lane == 0) {
+                    ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 0);
+                    if (ok) load_q(bt, sd, sm, l, g, false);
+                }
+                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
+                ++qn;
+                prev = key;
+            }
+            const int64_t c0 = (int64_t)un.c * kChunk1;
+            const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
+            for (int tile = 0; tile < nt; ++tile) {
+                if (lane == 0) ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 1);
+                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
+                const int64_t t_start = c0 + (int64_t)tile * kTileRows;
+                copy_tile_paged(sd, sm.k + (size_t)st * kTileBytes, l, g, [&](int r) { return t_start + r; },
+                                lane, bt.err);
+                paged_publish(ctl, stages, pub, ++kt, lag, lane);
+                if (++st == stages) { st = 0; ph ^= 1u; }
+            }
+        }
+        paged_publish(ctl, stages, pub, kt, 0, lane);
+        if (lane == 0 && qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
+    } else if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (elect_one()) {
             int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
@@ -568,7 +675,48 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
     my_range(bt.units2, &ub, &ue);
     const int stages = bt.stages;
 
-    if (warp == 0) {
+    if (warp == 0 && bt.paged) {
+        // ---------------- producer, paged cache: K rows by cp.async (whole warp) ----------------
+        const int lag = stages / 2;
+        int64_t kt = 0, pub = 0, qn = 0;   // tiles issued, tiles published, Q loads issued
+        int st = 0;
+        uint32_t ph = 0;
+        int prev = -1;
+        bool ok = true;
+        if (lane == 0) {
+            mbar_arrive_expect_tx(&ctl->o_full, 128 * 32);
+            tma_load_2d(sm.ones, &bt.omap, &ctl->o_full, 0, 0);
+        }
+        Unit un = decode2(bt, ub);
+        for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
+            const TcSender& sd = bt.s[un.i];
+            const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
+            const int key = un.i * 65536 + un.s;
+            if (key != prev) {
+                paged_publish(ctl, stages, pub, kt, 0, lane);   // q_empty needs the MMA past these
+                if (lane == 0) {
+                    ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 8);
+                    if (ok) load_q(bt, sd, sm, l, g, true);
+                }
+                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
+                ++qn;
+                prev = key;
+            }
+            if (lane == 0) ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 9);
+            if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
+            // quarter w of the tile (rows 32 w .. 32 w + 31) holds positions t0 + 26 w - 3 ..
+            const int64_t t0 = (int64_t)un.c * kOut2;
+            copy_tile_paged(sd, sm.k + (size_t)st * kTileBytes, l, g,
+                            [&](int r) { return t0 + kOutW * (r >> 5) - kMargin + (r & 31); }, lane, bt.err);
+            paged_publish(ctl, stages, pub, ++kt, lag, lane);
+            if (++st == stages) { st = 0; ph ^= 1u; }
+        }
+        paged_publish(ctl, stages, pub, kt, 0, lane);
+        if (lane == 0) {
+            if (qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
+            drain_wait(&ctl->o_full, 0);
+        }
+    } else if (warp == 0) {
         if (elect_one()) {
             int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
             int st = 0;               // ring slot of the next K tile and its phase parity
@@ -862,11 +1010,19 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
     // pattern), nothing has been launched and the caller uses the mma.sync passes.
     std::vector<TcBatch*> batches;
     auto free_all = [&] { for (TcBatch* p : batches) delete p; };
-    for (int b0 = 0; b0 < b.n; b0 += kMaxTcSenders) {
-        const int nb = b.n - b0 < kMaxTcSenders ? b.n - b0 : kMaxTcSenders;
+    // sub-batches of at most kMaxTcSenders consecutive senders of one layout (strided: K by
+    // TMA; paged: K by the producer warp's cp.async)
+    std::vector<int> firsts;
+    for (int b0 = 0; b0 < b.n;) {
+        int nb = 1;
+        const bool paged = b.s[b0].pm.pages != nullptr;
+        while (b0 + nb < b.n && nb < kMaxTcSenders && (b.s[b0 + nb].pm.pages != nullptr) == paged) ++nb;
+        firsts.push_back(b0);
         TcBatch* tb = new TcBatch();
         batches.push_back(tb);
+        tb->paged = paged ? 1 : 0;
         tb->n = nb;
+        b0 += nb;
         tb->nL = b.n_layers;
         tb->Hq = b.n_q_heads;
         tb->Hkv = b.n_kv_heads;
@@ -879,10 +1035,16 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         tb->err = err;
         int rpad_max = 128;
         int64_t u1 = 0, u2 = 0;
+        const int b_first = firsts.back();
         for (int k = 0; k < nb; ++k) {
-            const ScoreSender& s = b.s[b0 + k];
+            const ScoreSender& s = b.s[b_first + k];
             TcSender& d = tb->s[k];
             d.T = s.T;
+            d.k = s.k;
+            d.ks_l = s.ks_l;
+            d.ks_h = s.ks_h;
+            d.ks_p = s.ks_p;
+            d.pm = s.pm;
             d.m = s.m;
             d.inv_m = 1.f / (float)s.m;
             d.inv_mh = 1.f / ((float)s.m * (float)b.n_kv_heads);
@@ -920,8 +1082,9 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             const cuuint64_t ed[3] = {(cuuint64_t)kExtCols, (cuuint64_t)d.R_pad, (cuuint64_t)nS};
             const cuuint64_t es[2] = {(cuuint64_t)kExtCols * 2, (cuuint64_t)d.R_pad * kExtCols * 2};
             const cuuint32_t ebox[3] = {(cuuint32_t)kExtCols, (cuuint32_t)d.ebox_rows, 1};
-            if (!encode_4d(&d.kmap, s.k, kd, ks, kbox) || !encode_4d(&d.kmap32, s.k, kd, ks, kbox32) ||
-                !encode_4d(&d.qmap, s.q, qd, qs, qbox) || d.n_ebox * d.ebox_rows != d.R_pad || !b.ext ||
+            const bool kmaps_ok = paged || (encode_4d(&d.kmap, s.k, kd, ks, kbox) &&
+                                            encode_4d(&d.kmap32, s.k, kd, ks, kbox32));
+            if (!kmaps_ok || !encode_4d(&d.qmap, s.q, qd, qs, qbox) || d.n_ebox * d.ebox_rows != d.R_pad || !b.ext ||
                 !encode_nd(&d.emap, b.ext + s.ext_off, 3, ed, es, ebox, CU_TENSOR_MAP_SWIZZLE_32B)) {
                 free_all();
                 return cudaErrorNotSupported;
@@ -942,7 +1105,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
     cudaError_t e = cudaSuccess;
     for (size_t k = 0; k < batches.size() && e == cudaSuccess; ++k) {
         TcBatch* tb = batches[k];
-        const int b0 = (int)k * kMaxTcSenders;
+        const int b0 = firsts[k];
         const size_t smem = smem_bytes(tb->rpad_max, tb->stages);
         e = cudaFuncSetAttribute(k_stats_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e == cudaSuccess) {
