@@ -149,12 +149,19 @@ cb_status cb_create(const cb_config *cfg, cb_ctx **out);
  * b_{s,r,t} = mean of a over the G query heads of KV group s = (l, g); C = 1 where the
  * denominator is 0 (or below FLT_MIN in fp32).  Sender i is scored against queries[i].
  * Entries may repeat one sender cache with different queries: one launch then scores one
- * sender state against many receiver queries (multi-query serving: Sec. 5, Discussion, notes that one
- * completed sender state can be scored for several receiver queries), each pair exactly as if
- * it were scored alone.
+ * sender state against many receiver queries (multi-query serving: Sec. 5, Discussion, notes
+ * that one completed sender state can be scored for several receiver queries), each pair
+ * exactly as if it were scored alone.
+ * Paged senders (cb_kv.pages) on the tcgen05 passes are first copied into a contiguous staging
+ * buffer of the context (the copy is timed with pass 1).  The first call that needs more room
+ * than the buffer has allocates it anew, which waits for the device: make such a call before
+ * capturing cb_score in a CUDA graph.  Its size is that of the largest paged cache of the call,
+ * or of all of them up to 2 GiB, whichever is larger (senders beyond it are scored in later
+ * launches that reuse the buffer).
  *   n         1..max_senders;  senders, queries, scores: host arrays of n entries
  *   scores[i] device float[T_i], written; 16-byte aligned
- * Errors: CB_EINVAL (null/misaligned pointers, strides), CB_ESHAPE (T_i or m_i above the limits).
+ * Errors: CB_EINVAL (null/misaligned pointers, strides), CB_ESHAPE (T_i or m_i above the limits),
+ * CB_ENOMEM (no room for the staging buffer).
  */
 cb_status cb_score(cb_ctx *ctx, int32_t n, const cb_kv *senders, const cb_query *queries,
                    float *const *scores, void *stream);
@@ -261,7 +268,8 @@ void cb_destroy(cb_ctx *ctx);
 /* Text of the context's most recent error ("" if none).  NULL ctx: the last cb_create failure. */
 const char *cb_last_error(const cb_ctx *ctx);
 
-/* Device scratch bytes the context holds (for capacity planning). */
+/* Device scratch bytes the context holds now (for capacity planning; grows when cb_score
+ * first stages paged caches). */
 int64_t cb_scratch_bytes(const cb_ctx *ctx);
 
 /* Which implementation of the two logit passes (App. C.1) the context's last cb_score launched:

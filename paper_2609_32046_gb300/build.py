@@ -20,7 +20,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_NAME = "libcacheback.so"
 LIB_PATH = os.path.join(PKG, LIB_NAME)
-SOURCES = ["cb_api.cu", "cb_score.cu", "cb_score_tc.cu", "cb_select.cu", "cb_compact.cu", "cb_gather.cu", "cb_rope.cu"]
+SOURCES = ["cb_api.cu", "cb_score.cu", "cb_score_tc.cu", "cb_select.cu", "cb_compact.cu", "cb_gather.cu", "cb_rope.cu",
+           "cb_depage.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
                      "-I", INCLUDE, "-I", CSRC]

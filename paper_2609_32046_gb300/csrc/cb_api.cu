@@ -57,6 +57,8 @@ struct cb_ctx {
     float* part = nullptr;
     float* fin = nullptr;
     float* span_keys = nullptr;
+    uint16_t* stage = nullptr;      // tcgen05 passes: contiguous copies of paged senders' K (on demand)
+    int64_t stage_elems = 0;
     uint32_t* err = nullptr;
     int64_t keys_per_sender = 0;
     int64_t scratch_bytes = 0;
@@ -291,6 +293,7 @@ void cb_destroy(cb_ctx* ctx) {
         cudaFree(ctx->part);
         cudaFree(ctx->fin);
         cudaFree(ctx->span_keys);
+        cudaFree(ctx->stage);
         cudaFree(ctx->err);
         delete ctx->timer;
     }
@@ -332,6 +335,32 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
     }
     cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
     const int nS = c.n_layers * c.n_kv_heads;
+    if (ctx->use_tc) {
+        // paged senders are copied into a contiguous staging buffer for the tensor-map passes:
+        // room for the largest one, and for the rest up to kStageBudget elements per sub-batch
+        int64_t largest = 0, sum = 0;
+        for (int i = 0; i < n; ++i)
+            if (senders[i].pages) {
+                const int64_t e = (int64_t)nS * senders[i].T * c.head_dim;
+                largest = e > largest ? e : largest;
+                sum += e;
+            }
+        const int64_t want = largest > (sum < cbk::kStageBudget ? sum : cbk::kStageBudget)
+                                 ? largest : (sum < cbk::kStageBudget ? sum : cbk::kStageBudget);
+        if (want > ctx->stage_elems) {
+            cudaFree(ctx->stage);   // waits for work still using it
+            ctx->scratch_bytes -= ctx->stage_elems * 2;
+            ctx->stage = nullptr;
+            ctx->stage_elems = 0;
+            if (cudaMalloc(reinterpret_cast<void**>(&ctx->stage), (size_t)want * 2) != cudaSuccess) {
+                cudaGetLastError();
+                ctx->stage = nullptr;
+                return fail(ctx, CB_ENOMEM, "cannot allocate %lld bytes to stage paged caches", (long long)want * 2);
+            }
+            ctx->stage_elems = want;
+            ctx->scratch_bytes += want * 2;
+        }
+    }
     for (int b0 = 0; b0 < n; b0 += cbk::kMaxBatch) {
         const int nb = n - b0 < cbk::kMaxBatch ? n - b0 : cbk::kMaxBatch;
         cbk::ScoreBatch* bt = new cbk::ScoreBatch();
@@ -354,6 +383,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->ones = ctx->ones;
         bt->part = ctx->part;
         bt->fin = ctx->fin;
+        bt->stage = ctx->stage;
+        bt->stage_elems = ctx->stage_elems;
         int64_t so = 0, oo = 0, eo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];

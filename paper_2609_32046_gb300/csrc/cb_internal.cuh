@@ -95,7 +95,26 @@ struct ScoreBatch {
     const uint16_t* ones;     // tcgen05 passes: [128][16] bf16, columns 0-2 = 1, the rest 0
     float* part;              // per-group U_s, N_s, D_s partials
     float* fin;               // finalize slice sums [sender][kFinSlices][3][T]
+    uint16_t* stage;          // tcgen05 passes: contiguous copies of paged senders' K
+    int64_t stage_elems;      // its capacity (bf16 elements)
     ScoreSender s[kMaxBatch];
+};
+
+// Contiguous copy of paged caches: out[l][g][t][:] = K[l][g][t][:] read through the block table.
+constexpr int kMaxDepage = 32;
+struct DepageSender {
+    const uint16_t* k;        // the paged cache
+    int64_t ks_l, ks_h, ks_p;
+    PageMap pm;
+    int64_t T;
+    uint16_t* out;            // [nL][Hkv][T][128]
+};
+
+struct DepageBatch {
+    int32_t n;
+    int32_t n_layers, n_kv_heads;
+    uint32_t* err;
+    DepageSender s[kMaxDepage];
 };
 
 constexpr int kExtCols = 16;   // one bf16 K-step: the extra contraction column block of pass 2
@@ -173,6 +192,11 @@ cudaError_t launch_score(const ScoreBatch& b, cudaStream_t st, int num_sms, int*
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st);
 cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms);
 cudaError_t launch_gather(const GatherBatch& b, cudaStream_t st, int num_sms);
+// head_dim = 128 only (the tcgen05 passes' shape).
+cudaError_t launch_depage(const DepageBatch& b, cudaStream_t st, int num_sms);
+// Staging elements the tcgen05 passes want for paged senders (0 when none is paged): enough
+// for the largest paged sender and for paged sub-batches up to kStageBudget elements.
+constexpr int64_t kStageBudget = int64_t(1) << 30;
 // cb_compact with K rotated from sender position idx[j] to receiver position pos0 + out_off + j.
 cudaError_t launch_compact_rope(const CompactBatch& b, double base, int style, int64_t pos0, cudaStream_t st,
                                 int num_sms);

@@ -3,9 +3,10 @@
 // Both passes contract the receiver query Q_s = [(r, h) rows x d] of one KV group
 // s = (l, g) with that group's keys K_s = [positions x d] (App. C.1: a_{l,h,r,t} is the
 // softmax over t of scale * <q, k>).  Operands are K-major bf16 tiles in the 128-byte
-// swizzled layout, staged by TMA (or, for a paged cache, by the producer warp's cp.async);
-// one thread issues tcgen05.mma (fp32 accumulation in TMEM); the epilogue warps read TMEM
-// with tcgen05.ld.
+// swizzled layout, staged by TMA; one thread issues tcgen05.mma (fp32 accumulation in TMEM);
+// the epilogue warps read TMEM with tcgen05.ld.  A paged sender cache is first copied into a
+// contiguous staging buffer by k_depage (TMA needs a fixed tile shape, which a page boundary
+// inside a tile breaks), and both passes read that copy.
 //
 //   k_stats_tc  pass 1, D = Q_s K_tile^T: TMEM lane = row (r, h), column = position.
 //               Each epilogue thread owns one row and keeps its running max and
@@ -67,10 +68,6 @@ struct TcSender {
     int32_t ebox_rows, n_ebox;
     float inv_m, inv_mh;  // 1 / m and 1 / (m Hkv)
     int64_t unit1_begin, unit2_begin;
-    // paged cache (batches with paged != 0): K rows are copied by the producer warp
-    const uint16_t* k;
-    int64_t ks_l, ks_h, ks_p;
-    PageMap pm;
 };
 
 struct TcBatch {
@@ -80,12 +77,10 @@ struct TcBatch {
     int32_t stages, rpad_max;
     float sl2e, p;
     int32_t p_is_2, p_inf, ph;
-    int32_t paged;        // every sender of the batch has a block table (else none has)
     int64_t units1, units2;
     uint32_t* err;
     TcSender s[kMaxTcSenders];
 };
-static_assert(sizeof(TcBatch) <= 32000, "kernel parameter space");
 
 struct Ctl {
     uint64_t k_full[kMaxStages], k_empty[kMaxStages];
@@ -247,70 +242,6 @@ __device__ __forceinline__ void load_k(const TcSender& sd, const Smem& sm, int s
     tma_load_4d(dst + kTileBytes / 2, &sd.kmap, &sm.ctl->k_full[stage], 64, t_start, g, l);
 }
 
-// ---------------------------------------------------------------------------
-// Paged cache: the producer warp copies K tiles with cp.async.  Row r of a tile holds position
-// pos(r) (zero outside [0, T) and for a block-table entry outside the pool, which is recorded
-// in the error word), in the layout the TMA path writes: 64-column block kb at kb * 16 KB,
-// row r at r * 128 B, 16-byte piece j at (j ^ (r & 7)) * 16 (the 128-byte swizzle).
-// Completion runs through cp.async groups, one per tile: after committing tile k the warp
-// waits until `lag` groups at most are in flight, so tile k - lag has landed; each lane then
-// fences its writes into the async proxy that tcgen05.mma reads through, and lane 0 arrives
-// on the tile's k_full barrier (count 1, no transaction bytes).  Tiles held back this way
-// must all be published before the producer waits for the MMA issuer (q_empty), which
-// releases Q only after consuming every tile of the previous group.
-// ---------------------------------------------------------------------------
-template <typename Pos>
-__device__ __forceinline__ void copy_tile_paged(const TcSender& sd, uint8_t* dst, int l, int g, Pos pos, int lane,
-                                                uint32_t* err) {
-    const uint16_t* base = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
-    int64_t ro[4];   // element offsets of rows lane, lane + 32, lane + 64, lane + 96 (-1: zero row)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int64_t t = pos(q * 32 + lane);
-        ro[q] = -1;
-        if (t >= 0 && t < sd.T) {
-            ro[q] = row_offset(sd.pm, sd.ks_p, t);
-            if (ro[q] < 0) atomicOr(err, kErrPageIndex);
-        }
-    }
-    // lanes 0-15 copy the 16 pieces of row 2i, lanes 16-31 those of row 2i + 1
-    const int hr = lane >> 4, piece = lane & 15, kb = piece >> 3, j = piece & 7;
-    const uint32_t d0 = smem_u32(dst) + (uint32_t)kb * (kTileBytes / 2);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-#pragma unroll 4
-        for (int i = 0; i < 16; ++i) {
-            const int r = q * 32 + 2 * i + hr;
-            const int64_t o = __shfl_sync(0xffffffffu, ro[q], 2 * i + hr);
-            const uint32_t d = d0 + (uint32_t)r * 128u + ((uint32_t)(j ^ (r & 7)) << 4);
-            if (o >= 0)
-                cp_async16_zfill(d, base + o + kb * 64 + j * 8, 16u);
-            else
-                cp_async16_zfill(d, base, 0u);
-        }
-    }
-    cp_async_commit();
-}
-
-// Publish tiles [pub, kt - keep): wait until at most `keep` (0, 1 or 2) of this thread's groups
-// are in flight, fence, and arrive on their k_full barriers.  The producer keeps `lag` tiles in
-// flight in steady state and publishes everything (keep = 0) before it waits on anything the
-// MMA issuer releases only after consuming those tiles (q_empty), and at the end.
-__device__ __forceinline__ void paged_publish(Ctl* ctl, int stages, int64_t& pub, int64_t kt, int keep, int lane) {
-    if (kt - pub <= keep) return;
-    if (keep >= 2)
-        cp_async_wait<2>();
-    else if (keep == 1)
-        cp_async_wait<1>();
-    else
-        cp_async_wait<0>();
-    fence_proxy_async();
-    __syncwarp();
-    if (lane == 0)
-        for (int64_t k = pub; k < kt - keep; ++k) mbar_arrive(&ctl->k_full[k % stages]);
-    pub = kt - keep;
-}
-
 // One K = 128 contraction (8 UMMA K-steps).  a_base / b_base: first column block of each
 // operand (rows of 128 B); the second column block sits `a_blk` / `b_blk` bytes later.
 // The descriptors are built once; a K-step only moves the start-address field.
@@ -388,44 +319,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     my_range(bt.units1, &ub, &ue);
     const int stages = bt.stages;
 
-    if (warp == 0 && bt.paged) {
-        // ---------------- producer, paged cache: K rows by cp.async (whole warp) ----------------
-        const int lag = stages / 2;
-        int64_t kt = 0, pub = 0, qn = 0;   // tiles issued, tiles published, Q loads issued
-        int st = 0;
-        uint32_t ph = 0;
-        int prev = -1;
-        bool ok = true;
-        Unit un = decode1(bt, ub);
-        for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
-            const TcSender& sd = bt.s[un.i];
-            const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
-            const int key = un.i * 65536 + un.s;
-            if (key != prev) {
-                paged_publish(ctl, stages, pub, kt, 0, lane);   // q_empty needs the MMA past these
-                if (lane == 0) {
-                    ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 0);
-                    if (ok) load_q(bt, sd, sm, l, g, false);
-                }
-                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
-                ++qn;
-                prev = key;
-            }
-            const int64_t c0 = (int64_t)un.c * kChunk1;
-            const int nt = (int)((min((int64_t)kChunk1, sd.T - c0) + kTileRows - 1) / kTileRows);
-            for (int tile = 0; tile < nt; ++tile) {
-                if (lane == 0) ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 1);
-                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
-                const int64_t t_start = c0 + (int64_t)tile * kTileRows;
-                copy_tile_paged(sd, sm.k + (size_t)st * kTileBytes, l, g, [&](int r) { return t_start + r; },
-                                lane, bt.err);
-                paged_publish(ctl, stages, pub, ++kt, lag, lane);
-                if (++st == stages) { st = 0; ph ^= 1u; }
-            }
-        }
-        paged_publish(ctl, stages, pub, kt, 0, lane);
-        if (lane == 0 && qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
-    } else if (warp == 0) {
+    if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (elect_one()) {
             int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
@@ -675,48 +569,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
     my_range(bt.units2, &ub, &ue);
     const int stages = bt.stages;
 
-    if (warp == 0 && bt.paged) {
-        // ---------------- producer, paged cache: K rows by cp.async (whole warp) ----------------
-        const int lag = stages / 2;
-        int64_t kt = 0, pub = 0, qn = 0;   // tiles issued, tiles published, Q loads issued
-        int st = 0;
-        uint32_t ph = 0;
-        int prev = -1;
-        bool ok = true;
-        if (lane == 0) {
-            mbar_arrive_expect_tx(&ctl->o_full, 128 * 32);
-            tma_load_2d(sm.ones, &bt.omap, &ctl->o_full, 0, 0);
-        }
-        Unit un = decode2(bt, ub);
-        for (int64_t u = ub; u < ue && ok; ++u, next2(bt, un)) {
-            const TcSender& sd = bt.s[un.i];
-            const int l = un.s / bt.Hkv, g = un.s % bt.Hkv;
-            const int key = un.i * 65536 + un.s;
-            if (key != prev) {
-                paged_publish(ctl, stages, pub, kt, 0, lane);   // q_empty needs the MMA past these
-                if (lane == 0) {
-                    ok = wait_bar(&ctl->q_empty, (uint32_t)((qn & 1) ^ 1), ctl, bt.err, 8);
-                    if (ok) load_q(bt, sd, sm, l, g, true);
-                }
-                if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
-                ++qn;
-                prev = key;
-            }
-            if (lane == 0) ok = wait_bar(&ctl->k_empty[st], ph ^ 1u, ctl, bt.err, 9);
-            if (!(ok = __shfl_sync(0xffffffffu, ok, 0))) break;
-            // quarter w of the tile (rows 32 w .. 32 w + 31) holds positions t0 + 26 w - 3 ..
-            const int64_t t0 = (int64_t)un.c * kOut2;
-            copy_tile_paged(sd, sm.k + (size_t)st * kTileBytes, l, g,
-                            [&](int r) { return t0 + kOutW * (r >> 5) - kMargin + (r & 31); }, lane, bt.err);
-            paged_publish(ctl, stages, pub, ++kt, lag, lane);
-            if (++st == stages) { st = 0; ph ^= 1u; }
-        }
-        paged_publish(ctl, stages, pub, kt, 0, lane);
-        if (lane == 0) {
-            if (qn > 0) drain_wait(&ctl->q_full, (uint32_t)((qn - 1) & 1));
-            drain_wait(&ctl->o_full, 0);
-        }
-    } else if (warp == 0) {
+    if (warp == 0) {
         if (elect_one()) {
             int64_t kt = 0, qn = 0;   // K tiles and Q loads issued
             int st = 0;               // ring slot of the next K tile and its phase parity
@@ -1010,17 +863,35 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
     // pattern), nothing has been launched and the caller uses the mma.sync passes.
     std::vector<TcBatch*> batches;
     auto free_all = [&] { for (TcBatch* p : batches) delete p; };
-    // sub-batches of at most kMaxTcSenders consecutive senders of one layout (strided: K by
-    // TMA; paged: K by the producer warp's cp.async)
+    // Sub-batches of at most kMaxTcSenders senders; paged senders are first copied into the
+    // staging buffer (contiguous [nL][Hkv][T][128]), which each sub-batch reuses from its start,
+    // so a sub-batch also ends where its paged senders would overflow the staging.
     std::vector<int> firsts;
+    std::vector<DepageBatch*> depages;
+    auto free_depages = [&] { for (DepageBatch* p : depages) delete p; };
     for (int b0 = 0; b0 < b.n;) {
-        int nb = 1;
-        const bool paged = b.s[b0].pm.pages != nullptr;
-        while (b0 + nb < b.n && nb < kMaxTcSenders && (b.s[b0 + nb].pm.pages != nullptr) == paged) ++nb;
+        int nb = 0;
+        int64_t used = 0;
+        while (b0 + nb < b.n && nb < kMaxTcSenders) {
+            const ScoreSender& s = b.s[b0 + nb];
+            const int64_t e = s.pm.pages ? (int64_t)b.n_layers * b.n_kv_heads * s.T * 128 : 0;
+            if (e > 0 && (!b.stage || e > b.stage_elems)) {   // no room: the mma.sync passes read pages
+                free_all();
+                free_depages();
+                return cudaErrorNotSupported;
+            }
+            if (nb > 0 && used + e > b.stage_elems) break;
+            used += e;
+            ++nb;
+        }
         firsts.push_back(b0);
+        DepageBatch* dp = new DepageBatch();
+        depages.push_back(dp);
+        dp->n_layers = b.n_layers;
+        dp->n_kv_heads = b.n_kv_heads;
+        dp->err = err;
         TcBatch* tb = new TcBatch();
         batches.push_back(tb);
-        tb->paged = paged ? 1 : 0;
         tb->n = nb;
         b0 += nb;
         tb->nL = b.n_layers;
@@ -1034,17 +905,30 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         tb->ph = b.pool_half;
         tb->err = err;
         int rpad_max = 128;
-        int64_t u1 = 0, u2 = 0;
+        int64_t u1 = 0, u2 = 0, staged = 0;
         const int b_first = firsts.back();
         for (int k = 0; k < nb; ++k) {
             const ScoreSender& s = b.s[b_first + k];
             TcSender& d = tb->s[k];
+            // K as the passes read it: the sender's own tensor, or its staged copy
+            const uint16_t* kp = s.k;
+            int64_t kl = s.ks_l, kh = s.ks_h, kpos = s.ks_p;
+            if (s.pm.pages) {
+                DepageSender& ds = dp->s[dp->n++];
+                ds.k = s.k;
+                ds.ks_l = s.ks_l;
+                ds.ks_h = s.ks_h;
+                ds.ks_p = s.ks_p;
+                ds.pm = s.pm;
+                ds.T = s.T;
+                ds.out = b.stage + staged;
+                kp = ds.out;
+                kpos = 128;
+                kh = s.T * 128;
+                kl = (int64_t)b.n_kv_heads * s.T * 128;
+                staged += kl * b.n_layers;
+            }
             d.T = s.T;
-            d.k = s.k;
-            d.ks_l = s.ks_l;
-            d.ks_h = s.ks_h;
-            d.ks_p = s.ks_p;
-            d.pm = s.pm;
             d.m = s.m;
             d.inv_m = 1.f / (float)s.m;
             d.inv_mh = 1.f / ((float)s.m * (float)b.n_kv_heads);
@@ -1067,10 +951,11 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             d.n_qbox = tok_pad / d.qbox_tok;
             if (d.n_qbox * d.qbox_tok != tok_pad) {
                 free_all();
+                free_depages();
                 return cudaErrorNotSupported;
             }
             const cuuint64_t kd[4] = {128, (cuuint64_t)s.T, (cuuint64_t)b.n_kv_heads, (cuuint64_t)b.n_layers};
-            const cuuint64_t ks[3] = {(cuuint64_t)s.ks_p * 2, (cuuint64_t)s.ks_h * 2, (cuuint64_t)s.ks_l * 2};
+            const cuuint64_t ks[3] = {(cuuint64_t)kpos * 2, (cuuint64_t)kh * 2, (cuuint64_t)kl * 2};
             const cuuint32_t kbox[4] = {64, kTileRows, 1, 1};
             const cuuint64_t qd[4] = {128, (cuuint64_t)b.n_q_heads, (cuuint64_t)s.m, (cuuint64_t)b.n_layers};
             const cuuint64_t qs[3] = {(cuuint64_t)s.qs_h * 2, (cuuint64_t)s.qs_t * 2, (cuuint64_t)s.qs_l * 2};
@@ -1082,11 +967,11 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
             const cuuint64_t ed[3] = {(cuuint64_t)kExtCols, (cuuint64_t)d.R_pad, (cuuint64_t)nS};
             const cuuint64_t es[2] = {(cuuint64_t)kExtCols * 2, (cuuint64_t)d.R_pad * kExtCols * 2};
             const cuuint32_t ebox[3] = {(cuuint32_t)kExtCols, (cuuint32_t)d.ebox_rows, 1};
-            const bool kmaps_ok = paged || (encode_4d(&d.kmap, s.k, kd, ks, kbox) &&
-                                            encode_4d(&d.kmap32, s.k, kd, ks, kbox32));
-            if (!kmaps_ok || !encode_4d(&d.qmap, s.q, qd, qs, qbox) || d.n_ebox * d.ebox_rows != d.R_pad || !b.ext ||
+            if (!encode_4d(&d.kmap, kp, kd, ks, kbox) || !encode_4d(&d.kmap32, kp, kd, ks, kbox32) ||
+                !encode_4d(&d.qmap, s.q, qd, qs, qbox) || d.n_ebox * d.ebox_rows != d.R_pad || !b.ext ||
                 !encode_nd(&d.emap, b.ext + s.ext_off, 3, ed, es, ebox, CU_TENSOR_MAP_SWIZZLE_32B)) {
                 free_all();
+                free_depages();
                 return cudaErrorNotSupported;
             }
         }
@@ -1095,6 +980,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         const cuuint32_t obox[2] = {(cuuint32_t)kExtCols, 128};
         if (!encode_nd(&tb->omap, b.ones, 2, od, os, obox, CU_TENSOR_MAP_SWIZZLE_32B)) {
             free_all();
+            free_depages();
             return cudaErrorNotSupported;
         }
         tb->rpad_max = rpad_max;
@@ -1109,8 +995,11 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         const size_t smem = smem_bytes(tb->rpad_max, tb->stages);
         e = cudaFuncSetAttribute(k_stats_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e == cudaSuccess) {
-            const int g1 = (int)(tb->units1 < num_sms ? tb->units1 : num_sms);
             stage_mark(b.timer, kStageStart, st);
+            e = launch_depage(*depages[k], st, num_sms);   // timed with pass 1
+        }
+        if (e == cudaSuccess) {
+            const int g1 = (int)(tb->units1 < num_sms ? tb->units1 : num_sms);
             k_stats_tc<<<g1, kThreadsTc, smem, st>>>(*tb);
             stage_mark(b.timer, kStageStats, st);
             e = cudaGetLastError();
@@ -1136,6 +1025,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         }
     }
     free_all();
+    free_depages();
     return e;
 }
 

@@ -113,27 +113,6 @@ __device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* m, int32_t
 }
 
 // ---------------------------------------------------------------------------
-// cp.async (per-thread 16-byte copies; used where rows have no tensor-map shape, e.g. a
-// paged cache).  Their shared-memory writes belong to the generic proxy: the writing thread
-// must wait for them and issue fence_proxy_async() before an async-proxy reader (tcgen05.mma,
-// TMA) may use the data.
-// ---------------------------------------------------------------------------
-// 16 bytes from gmem to smem; src_bytes < 16 zero-fills the rest (0: nothing is read).
-__device__ __forceinline__ void cp_async16_zfill(uint32_t smem, const void* gmem, uint32_t src_bytes) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem), "l"(gmem), "r"(src_bytes) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-
-// Wait until at most N of this thread's committed groups are still in flight.
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
-// ---------------------------------------------------------------------------
 // tcgen05: tensor memory
 // ---------------------------------------------------------------------------
 // Allocate `ncols` TMEM columns (power of two >= 32); the address is written to *slot.  Whole warp.
