@@ -6,8 +6,8 @@
 //   pass 2  k_accum     per (sender, s, 128-position chunk + 8-position halo):
 //                       a/G = exp2(z - offset), b = sum over the group's heads,
 //                       N_s = sum_r Pool(b_r)^p, bsum = sum_r b  ->  U_s, N_s, D_s
-//   k_finalize          per (sender, 240-position tile): fixed-order sums over s,
-//                       Q = Pool(U), C = (N/D)^(1/(p-1)), S = Q * C^alpha
+//   k_finalize          per (sender, 240-position tile, slice of the groups): fixed-order
+//                       sums over s, Q = Pool(U), C = (N/D)^(1/(p-1)), S = Q * C^alpha
 //
 // Both logit passes use the bf16 tensor cores through mma.sync m16n8k16 with fp32
 // accumulation.  Rows of one m16 tile are (8 query tokens) x (2 heads of the
@@ -278,15 +278,24 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
     float M = -INFINITY, L = 0.f;
     if (row < R) {
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
-#pragma unroll 4
-        for (int c = j; c < sd.n_chunk1; c += 4) {
-            const float2 v = st[(int64_t)c * R];
-            if (v.x == -INFINITY) continue;
-            if (v.x > M) {
-                L = (M == -INFINITY ? 0.f : L * ex2(M - v.x)) + v.y;
-                M = v.x;
-            } else {
-                L += v.y * ex2(v.x - M);
+        // slots j, j + 4, j + 8, ... merged in that order; eight loads issued before each merge run
+        for (int c0 = j; c0 < sd.n_chunk1; c0 += 32) {
+            float2 vv[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int c = c0 + 4 * q;
+                vv[q] = c < sd.n_chunk1 ? st[(int64_t)c * R] : make_float2(-INFINITY, 0.f);
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const float2 v = vv[q];
+                if (v.x == -INFINITY) continue;
+                if (v.x > M) {
+                    L = (M == -INFINITY ? 0.f : L * ex2(M - v.x)) + v.y;
+                    M = v.x;
+                } else {
+                    L += v.y * ex2(v.x - M);
+                }
             }
         }
         if (sd.kself) {
@@ -480,68 +489,82 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 }
 
 // ---------------------------------------------------------------------------
-// finalize: fixed-order sums over the groups, Pool(U), C, S
+// finalize: fixed-order sums over the groups, Pool(U), C, S -- one launch
 // ---------------------------------------------------------------------------
-// Stage 1: slice k of the groups (s = k, k + 16, ...) summed in increasing order per position.
-__global__ void __launch_bounds__(256) k_fin_sum(const __grid_constant__ ScoreBatch bt) {
-    const int nS = bt.n_layers * bt.n_kv_heads;
-    const ScoreSender& sd = bt.s[blockIdx.z];
-    const int sl = blockIdx.y;
-    const int64_t T = sd.T;
-    const int64_t t = (int64_t)blockIdx.x * 256 + threadIdx.x;
-    if (t >= T) return;
-    const float* part = bt.part + sd.part_off + t;
-    float U = 0.f, Nv = 0.f, Dv = 0.f;   // p = infinity: N and D are maxima over the groups (all >= 0)
-    if (bt.p_inf) {
-#pragma unroll 6
-        for (int s = sl; s < nS; s += kFinSlices) {
-            U += __ldcs(part + (int64_t)s * T);
-            Nv = fmaxf(Nv, __ldcs(part + ((int64_t)nS + s) * T));
-            Dv = fmaxf(Dv, __ldcs(part + ((int64_t)2 * nS + s) * T));
-        }
-    } else {
-#pragma unroll 6
-        for (int s = sl; s < nS; s += kFinSlices) {
-            U += __ldcs(part + (int64_t)s * T);
-            Nv += __ldcs(part + ((int64_t)nS + s) * T);
-            Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
-        }
-    }
-    float* fin = bt.fin + sd.fin_off + (int64_t)sl * 3 * T + t;
-    fin[0] = U;
-    fin[T] = Nv;
-    fin[2 * T] = Dv;
-}
-
-// Stage 2: the 16 slice sums in fixed order, Pool(U) through shared memory, C and S.
+// Block (tile, slice k, sender) covers the tile's 256 positions: 240 outputs and kHalo on each
+// side for Pool.  It sums slice k of the groups (s = k, k + 16, ...) in increasing order per
+// position (U everywhere, N and D at the outputs) into the tile's slice buffer, then counts
+// itself done on the tile's counter.  The last of the tile's 16 slice blocks adds the 16 slice
+// sums in slice order, pools U and writes C and S, and resets the counter for the next call.
+// The order of every sum is fixed, so the result does not depend on which block is last.
 constexpr int kFinBlock = 256;
-constexpr int kFinOut2 = kFinBlock - 2 * kHalo;        // outputs per block
+constexpr int kFinOut2 = kFinBlock - 2 * kHalo;        // outputs per tile
 
 __global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ ScoreBatch bt) {
     __shared__ float us[kFinBlock];
-    const int64_t blk = blockIdx.x;
-    const int i = find_sender(bt.n, blk, [&](int k) { return bt.s[k].blkf_begin; });
-    const ScoreSender& sd = bt.s[i];
+    __shared__ int last;
+    const ScoreSender& sd = bt.s[blockIdx.z];
     const int64_t T = sd.T;
+    const int64_t tile = blockIdx.x;
+    if (tile * kFinOut2 >= T) return;
+    const int sl = blockIdx.y;
+    const int nS = bt.n_layers * bt.n_kv_heads;
     const int lp = threadIdx.x;
-    const int64_t t = (blk - sd.blkf_begin) * kFinOut2 - kHalo + lp;
+    const int64_t t = tile * kFinOut2 - kHalo + lp;
     const bool inside = (t >= 0 && t < T);
     const bool centre = lp >= kHalo && lp < kFinBlock - kHalo;
-    const float* fin = bt.fin + sd.fin_off + t;
+    float* fin = bt.fin + sd.fin_off + tile * (kFinSlices * 3 * kFinBlock);   // [slice][3][256]
+    {
+        float U = 0.f, Nv = 0.f, Dv = 0.f;   // p = infinity: N and D are maxima over the groups (all >= 0)
+        if (inside) {
+            const float* part = bt.part + sd.part_off + t;
+            if (!centre) {
+#pragma unroll 18
+                for (int s = sl; s < nS; s += kFinSlices) U += __ldcs(part + (int64_t)s * T);
+            } else if (bt.p_inf) {
+#pragma unroll 18
+                for (int s = sl; s < nS; s += kFinSlices) {
+                    U += __ldcs(part + (int64_t)s * T);
+                    Nv = fmaxf(Nv, __ldcs(part + ((int64_t)nS + s) * T));
+                    Dv = fmaxf(Dv, __ldcs(part + ((int64_t)2 * nS + s) * T));
+                }
+            } else {
+#pragma unroll 18
+                for (int s = sl; s < nS; s += kFinSlices) {
+                    U += __ldcs(part + (int64_t)s * T);
+                    Nv += __ldcs(part + ((int64_t)nS + s) * T);
+                    Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
+                }
+            }
+        }
+        float* f = fin + sl * 3 * kFinBlock + lp;
+        f[0] = U;
+        f[kFinBlock] = Nv;
+        f[2 * kFinBlock] = Dv;
+    }
+    __threadfence();
+    __syncthreads();
+    uint32_t* cnt = bt.fin_cnt + sd.blkf_begin + tile;
+    if (lp == 0) last = atomicAdd(cnt, 1u) == kFinSlices - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
     float U = 0.f, Nv = 0.f, Dv = 0.f;
     if (inside) {
 #pragma unroll
-        for (int k = 0; k < kFinSlices; ++k) U += fin[(int64_t)k * 3 * T];
+        for (int k = 0; k < kFinSlices; ++k) U += __ldcg(fin + k * 3 * kFinBlock + lp);
         if (centre) {
 #pragma unroll
             for (int k = 0; k < kFinSlices; ++k) {
-                const float n_k = fin[((int64_t)k * 3 + 1) * T], d_k = fin[((int64_t)k * 3 + 2) * T];
+                const float n_k = __ldcg(fin + (k * 3 + 1) * kFinBlock + lp);
+                const float d_k = __ldcg(fin + (k * 3 + 2) * kFinBlock + lp);
                 Nv = bt.p_inf ? fmaxf(Nv, n_k) : Nv + n_k;
                 Dv = bt.p_inf ? fmaxf(Dv, d_k) : Dv + d_k;
             }
         }
     }
     us[lp] = U;
+    if (lp == 0) *cnt = 0u;   // every slice block of this tile has counted itself
     __syncthreads();
     if (centre && inside) {
         const int ph = bt.pool_half;
@@ -553,15 +576,18 @@ __global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ 
     }
 }
 
+}  // namespace
+
+int64_t finalize_tiles(int64_t T) { return (T + kFinOut2 - 1) / kFinOut2; }
+int64_t finalize_floats(int64_t T) { return finalize_tiles(T) * kFinSlices * 3 * kFinBlock; }
+
+namespace {
+
 cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
-    int64_t maxT = 0, nblk = 0;
-    for (int i = 0; i < b.n; ++i) {
-        maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
-        nblk += (b.s[i].T + kFinOut2 - 1) / kFinOut2;
-    }
-    dim3 g1((unsigned)((maxT + 255) / 256), kFinSlices, (unsigned)b.n);
-    k_fin_sum<<<g1, 256, 0, st>>>(b);
-    k_finalize<<<(unsigned)nblk, kFinBlock, 0, st>>>(b);
+    int64_t maxT = 0;
+    for (int i = 0; i < b.n; ++i) maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
+    dim3 grid((unsigned)finalize_tiles(maxT), kFinSlices, (unsigned)b.n);
+    k_finalize<<<grid, kFinBlock, 0, st>>>(b);
     return cudaGetLastError();
 }
 
@@ -583,8 +609,6 @@ cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-int64_t finalize_blocks(int64_t T) { return (T + kFinOut2 - 1) / kFinOut2; }
-
 
 template <int D, int G>
 size_t accum_smem(int max_rows) {
@@ -600,7 +624,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     for (int i = 0; i < b.n; ++i) {
         nblk1 += (int64_t)nS * b.s[i].n_chunk1;
         nblk2 += (int64_t)nS * b.s[i].n_chunk2;
-        nblkf += finalize_blocks(b.s[i].T);
+        nblkf += finalize_tiles(b.s[i].T);
         max_rows = max_rows > b.s[i].m * G ? max_rows : b.s[i].m * G;
     }
     const size_t smem1 = (size_t)kStatsChunk * D * 2;
@@ -633,7 +657,7 @@ cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms, i
     int64_t bf = 0;
     for (int i = 0; i < bp->n; ++i) {
         bp->s[i].blkf_begin = bf;
-        bf += finalize_blocks(bp->s[i].T);
+        bf += finalize_tiles(bp->s[i].T);
     }
     const ScoreBatch& b = *bp;
     struct Free { ScoreBatch* p; ~Free() { delete p; } } guard{bp};

@@ -30,6 +30,14 @@ namespace {
 
 constexpr int kSelThreads = 1024;
 constexpr int kWarps = kSelThreads / 32;
+constexpr int kScoreTile = 8192;                       // scores staged in shared memory per step
+constexpr int kPadTile = kScoreTile + kScoreTile / 32;  // one pad word per 32 (span sums free of bank conflicts)
+constexpr int kPerThread = kScoreTile / kSelThreads;    // scores each thread stages per tile
+constexpr int kSmemSpans = 8192;     // span means kept in shared memory when there are at most this many
+// two score tiles, the span means, and (one span a thread) each span's [left, right] run
+constexpr size_t kSelDynSmem = (size_t)(2 * kPadTile + kSmemSpans + kSelThreads) * sizeof(float);
+
+__device__ __forceinline__ int pad(int k) { return k + (k >> 5); }
 
 __device__ __forceinline__ uint32_t order_key(float f) {
     const uint32_t u = __float_as_uint(f == 0.f ? 0.f : f);  // -0 ranks with +0
@@ -77,13 +85,17 @@ __device__ int64_t block_exclusive_scan(int64_t v, int64_t* sh, int64_t* total) 
 }
 
 __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ SelectBatch bt) {
-    __shared__ uint32_t hist[kWarps][256];
-    __shared__ int64_t hsum[256];
+    __shared__ uint32_t hist[256];
     __shared__ int64_t scan_sh[32];
     __shared__ float red[32];
+    __shared__ float head[kMaxSpanWidth];   // scores of the first span
     __shared__ int64_t sel_bucket, sel_before;
 
-    const SelectSender& sd = bt.s[blockIdx.x];
+    // this block's sender in shared memory: reads of the parameter array at a run-time index
+    // are slow, and with 64 registers a thread the compiler re-reads such values in loops
+    __shared__ SelectSender sd;
+    if (threadIdx.x == 0) sd = bt.s[blockIdx.x];
+    __syncthreads();
     const int64_t T = sd.T, B = sd.B;
     const int w = bt.span_w;
     const int64_t nsp = (T + w - 1) / w;
@@ -93,9 +105,52 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     F.a = bt.n_sink < T ? bt.n_sink : T;
     F.b = T - bt.n_latent > 0 ? T - bt.n_latent : 0;
 
-    // 1. maximum score and span means
+    // 1. maximum score and span means.  Scores pass through shared memory a tile of whole spans
+    // at a time (coalesced loads, two buffers: the next tile is loaded into registers while the
+    // current one is summed); each thread sums its spans there, in index order.  The first span
+    // (whose first score is replaced by the maximum) is summed last, once the maximum is known.
+    extern __shared__ float dsm[];
+    float* keys = nsp <= kSmemSpans ? dsm + 2 * kPadTile : sd.span_keys;
+    const bool sink = bt.n_sink > 0;
+    const int64_t tile = (int64_t)(kScoreTile / w) * w;     // whole spans per tile
+    const int64_t ntile = (T + tile - 1) / tile;
+    float nxt[kPerThread];
+#pragma unroll
+    for (int q = 0; q < kPerThread; ++q) {
+        const int k = tid + q * kSelThreads;
+        nxt[q] = k < tile && k < T ? S[k] : 0.f;
+    }
     float mx = -INFINITY;
-    for (int64_t t = tid; t < T; t += kSelThreads) mx = fmaxf(mx, S[t]);
+    for (int64_t it = 0; it < ntile; ++it) {
+        const int64_t t0 = it * tile, n = T - t0 < tile ? T - t0 : tile;
+        float* ts = dsm + (it & 1) * kPadTile;
+#pragma unroll
+        for (int q = 0; q < kPerThread; ++q) {
+            const int k = tid + q * kSelThreads;
+            if (k < n) {
+                ts[pad(k)] = nxt[q];
+                mx = fmaxf(mx, nxt[q]);
+                if (it == 0 && k < w) head[k] = nxt[q];
+            }
+        }
+        __syncthreads();   // this tile is in place; the tile before the previous one is summed
+        if (it + 1 < ntile) {
+            const int64_t t1 = t0 + tile, n1 = T - t1 < tile ? T - t1 : tile;
+#pragma unroll
+            for (int q = 0; q < kPerThread; ++q) {
+                const int k = tid + q * kSelThreads;
+                nxt[q] = k < n1 ? S[t1 + k] : 0.f;
+            }
+        }
+        const int64_t ja = t0 / w, jb = (t0 + n + w - 1) / w;
+        for (int64_t j = ja + tid; j < jb; j += kSelThreads) {
+            if (j == 0 && sink) continue;
+            const int lo = (int)(j * w - t0), hi = (int)((j * w + w < T ? j * w + w : T) - t0);
+            float acc = 0.f;
+            for (int k = lo; k < hi; ++k) acc += ts[pad(k)];
+            keys[j] = __fdiv_rn(acc, (float)(hi - lo));
+        }
+    }
 #pragma unroll
     for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     if (lane == 0) red[warp] = mx;
@@ -108,12 +163,14 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     }
     __syncthreads();
     const float smax = red[0];
-    for (int64_t j = tid; j < nsp; j += kSelThreads) {
-        const int64_t lo = j * w, hi = lo + w < T ? lo + w : T;
+    if (sink && tid == 0) {
+        const int hi = w < T ? w : (int)T;
         float acc = 0.f;
-        for (int64_t t = lo; t < hi; ++t) acc += (t == 0 && bt.n_sink > 0) ? smax : S[t];
-        sd.span_keys[j] = __fdiv_rn(acc, (float)(hi - lo));
+        for (int k = 0; k < hi; ++k) acc += k == 0 ? smax : head[k];
+        keys[0] = __fdiv_rn(acc, (float)hi);
     }
+    // a single tile still holds every score (the partial span's best position is looked up there)
+    const float* all_s = ntile == 1 ? dsm : nullptr;
     const int64_t need = B - F.count(0, T);
     __syncthreads();
 
@@ -123,27 +180,21 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     if (need > 0) {
         for (int pass = 0; pass < 4; ++pass) {
             const int shift = 24 - 8 * pass;
-            for (int k = tid; k < kWarps * 256; k += kSelThreads) (&hist[0][0])[k] = 0u;
+            if (tid < 256) hist[tid] = 0u;
             __syncthreads();
             for (int64_t j = tid; j < nsp; j += kSelThreads) {
-                const uint32_t key = order_key(sd.span_keys[j]);
+                const uint32_t key = order_key(keys[j]);
                 if ((key & pmask) != prefix) continue;
                 const int64_t lo = j * w, hi = lo + w < T ? lo + w : T;
                 const uint32_t u = (uint32_t)((hi - lo) - F.count(lo, hi));
-                if (u) atomicAdd(&hist[warp][(key >> shift) & 255u], u);
-            }
-            __syncthreads();
-            if (tid < 256) {
-                int64_t v = 0;
-                for (int k = 0; k < kWarps; ++k) v += hist[k][tid];
-                hsum[tid] = v;
+                if (u) atomicAdd(&hist[(key >> shift) & 255u], u);
             }
             __syncthreads();
             if (warp == 0) {
                 // lane L owns buckets 255-8L .. 248-8L (descending key order)
                 int64_t mine = 0;
 #pragma unroll
-                for (int k = 0; k < 8; ++k) mine += hsum[255 - 8 * lane - k];
+                for (int k = 0; k < 8; ++k) mine += hist[255 - 8 * lane - k];
                 int64_t incl = mine;
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) {
@@ -157,8 +208,8 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
                     int64_t before = excl;
                     for (int k = 0; k < 8; ++k) {
                         const int bucket = 255 - 8 * lane - k;
-                        if (before + hsum[bucket] >= rem) { sel_bucket = bucket; sel_before = before; break; }
-                        before += hsum[bucket];
+                        if (before + hist[bucket] >= rem) { sel_bucket = bucket; sel_before = before; break; }
+                        before += hist[bucket];
                     }
                 }
             }
@@ -166,7 +217,6 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             prefix |= (uint32_t)sel_bucket << shift;
             pmask |= 255u << shift;
             rem -= sel_before;
-            __syncthreads();
         }
     }
     const uint32_t kappa = prefix;
@@ -178,7 +228,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     int64_t tie_mine = 0;
     if (need > 0)
         for (int64_t j = j0; j < j1; ++j)
-            if (order_key(sd.span_keys[j]) == kappa) {
+            if (order_key(keys[j]) == kappa) {
                 const int64_t lo = j * w, hi = lo + w < T ? lo + w : T;
                 tie_mine += (hi - lo) - F.count(lo, hi);
             }
@@ -192,7 +242,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             const int64_t f = F.count(lo, hi), u = (hi - lo) - f;
             int64_t take = 0;
             if (need > 0) {
-                const uint32_t key = order_key(sd.span_keys[j]);
+                const uint32_t key = order_key(keys[j]);
                 if (key > kappa) take = u;
                 else if (key == kappa) {
                     take = rem - tb;
@@ -207,7 +257,15 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     int64_t out = block_exclusive_scan(cnt_mine, scan_sh, &total);
     if (tid == 0 && total != B) atomicOr(bt.err, kErrSelectBudget);
 
-    // 4. write positions in source order
+    // 4. write positions in source order.  Each thread settles what its spans contribute:
+    // everything, only the forced positions, or the forced ones plus the run [left, right]
+    // around the partial span's best position.  With one span a thread, a span's output start
+    // (in place of its mean, which is no longer needed) and its run go to shared memory and each
+    // warp then writes whole spans, 32 consecutive positions per step, so the stores are
+    // coalesced; with several (measured faster that way), every thread writes its own spans.
+    const bool coop = nsp <= kSelThreads;   // one span a thread (more: each thread writes its own)
+    int32_t* span_at = reinterpret_cast<int32_t*>(keys);
+    int32_t* span_run = reinterpret_cast<int32_t*>(dsm + 2 * kPadTile + kSmemSpans);
     {
         int64_t tb = tie_before;
         for (int64_t j = j0; j < j1; ++j) {
@@ -215,7 +273,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             const int64_t f = F.count(lo, hi), u = (hi - lo) - f;
             int64_t take = 0;
             if (need > 0) {
-                const uint32_t key = order_key(sd.span_keys[j]);
+                const uint32_t key = order_key(keys[j]);
                 if (key > kappa) take = u;
                 else if (key == kappa) {
                     take = rem - tb;
@@ -223,20 +281,25 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
                     tb += u;
                 }
             }
+            int64_t left = lo, right = lo - 1;   // empty run: only the forced positions
             if (take == u) {
-                for (int64_t t = lo; t < hi; ++t)
-                    if (out < B) sd.idx[out++] = (int32_t)t;
-            } else if (take == 0) {
-                for (int64_t t = lo; t < hi; ++t)
-                    if (F.at(t) && out < B) sd.idx[out++] = (int32_t)t;
-            } else {
+                left = lo;
+                right = hi - 1;
+            } else if (take > 0) {
                 // highest-scoring unforced position (lowest index on ties)
                 int64_t c = -1;
+                float best = 0.f;
                 for (int64_t t = lo; t < hi; ++t)
-                    if (!F.at(t) && (c < 0 || S[t] > S[c])) c = t;
+                    if (!F.at(t)) {
+                        const float v = all_s ? all_s[pad((int)t)] : S[t];
+                        if (c < 0 || v > best) {
+                            c = t;
+                            best = v;
+                        }
+                    }
                 // grow a run of unforced positions around c, nearer first, lower index on ties
-                int64_t left = c, right = c, got = 1;
-                int64_t nl = c - 1, nr = c + 1;
+                int64_t got = 1, nl = c - 1, nr = c + 1;
+                left = right = c;
                 while (nl >= lo && F.at(nl)) --nl;
                 while (nr < hi && F.at(nr)) ++nr;
                 while (got < take) {
@@ -253,8 +316,37 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
                     }
                     ++got;
                 }
+            }
+            if (coop) {
+                span_at[j] = (int32_t)out;   // B < 2^31
+                span_run[j] = (int32_t)((left - lo + 1) | ((right - lo + 1) << 16));
+            } else {
                 for (int64_t t = lo; t < hi; ++t)
-                    if ((F.at(t) || (t >= left && t <= right)) && out < B) sd.idx[out++] = (int32_t)t;
+                    if ((F.at(t) || (t >= left && t <= right)) && out < B) sd.idx[out] = (int32_t)t, ++out;
+                continue;
+            }
+            out += f + take;
+        }
+    }
+    if (coop) {
+        __syncthreads();
+        // 32-bit arithmetic throughout (T < 2^31): this loop is bound by instruction issue
+        const int32_t T32 = (int32_t)T, B32 = (int32_t)(B < T ? B : T), fa = (int32_t)F.a, fb = (int32_t)F.b;
+        const int32_t nsp32 = (int32_t)nsp;
+        const unsigned below = (1u << lane) - 1u;
+        int32_t* const idx = sd.idx;
+        for (int32_t j = warp; j < nsp32; j += kWarps) {
+            const int32_t lo = j * w, hi = lo + w < T32 ? lo + w : T32;
+            const int32_t run = span_run[j];
+            const int32_t left = lo + (run & 0xffff) - 1, right = lo + (run >> 16) - 1;
+            int32_t base = span_at[j];
+            for (int32_t c0 = lo; c0 < hi; c0 += 32) {
+                const int32_t t = c0 + lane;
+                const bool sel = t < hi && (t < fa || t >= fb || (t >= left && t <= right));
+                const unsigned m = __ballot_sync(0xffffffffu, sel);
+                const int32_t o = base + __popc(m & below);
+                if (sel && o < B32) idx[o] = t;
+                base += __popc(m);
             }
         }
     }
@@ -263,7 +355,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
 }  // namespace
 
 cudaError_t launch_select(const SelectBatch& b, cudaStream_t st) {
-    k_select<<<(unsigned)b.n, kSelThreads, 0, st>>>(b);
+    // per device (the attribute belongs to the current device's copy of the kernel)
+    const cudaError_t attr =
+        cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSelDynSmem);
+    if (attr != cudaSuccess) return attr;
+    k_select<<<(unsigned)b.n, kSelThreads, kSelDynSmem, st>>>(b);
     return cudaGetLastError();
 }
 
