@@ -244,6 +244,11 @@ def max_over_ranks(ws, x: float) -> float:
 # CPU oracle timing (the cpu_baseline object and the reference arm)
 # ---------------------------------------------------------------------------
 
+def synth_spec(name: str):
+    import synth
+    return synth.SPECS[name]
+
+
 def sample_layers(spec) -> int:
     """Layers of sender 0 the oracle scores per sample: all 36 for a Qwen3-8B-shaped sender of
     8192 positions and 64 query tokens (a few seconds on the host cores), proportionally fewer
@@ -314,8 +319,12 @@ def run_reference(args):
     import oracle
     oracle.build()
     vals = []
+    # each step a short sample (a ninth of the baseline's layers: ~0.3 s on 16 cores for
+    # qwen8b), so that --steps K --warmup W stays within a few minutes for the usual K
+    spec0 = synth_spec(args.workload)
+    layers = max(1, sample_layers(spec0) // 9) if not args.cpu_layers else args.cpu_layers
     for k in range(args.warmup + args.steps):
-        r = oracle_sample(args.workload)
+        r = oracle_sample(args.workload, layers)
         if k >= args.warmup:
             vals.append(r)
     v = statistics.median([x["value"] for x in vals])
