@@ -462,11 +462,18 @@ def run_ours(args):
 
     tokens_per_rank = sum(f.Ts)
     def launches(n):
-        # per call group of <= 64 senders: statistics, combine and accumulation per <= 32 senders,
-        # then the two finalize kernels; one select and one compact launch per <= 64 senders
+        # per call group of <= 64 senders: statistics, combine and accumulation per sub-batch of
+        # <= 32 senders (paged caches: also a de-page launch, and sub-batches end where the staging
+        # buffer is full), then one finalize launch; one select and one compact launch per group
         sb = math.ceil(n / 64)
-        tc = sum(math.ceil(min(64, n - 64 * b) / 32) for b in range(sb))
-        return 3 * tc + 2 * sb + sb + sb
+        if not args.paged:
+            tc = sum(math.ceil(min(64, n - 64 * b) / 32) for b in range(sb))
+            return 3 * tc + sb + sb + sb
+        e = spec.shape.n_layers * spec.shape.n_kv_heads * max(spec.T) * spec.shape.head_dim
+        stage = max(e, min(n * e, 1 << 30))
+        per = max(1, min(32, stage // e))
+        tc = sum(math.ceil(min(64, n - 64 * b) / per) for b in range(sb))
+        return 4 * tc + sb + sb + sb
 
     waves = [min(wave, n_send - a) for a in range(0, n_send, wave)] if wave else [n_send]
     launches_per_step = sum(launches(n) for n in waves)
