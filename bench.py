@@ -484,47 +484,76 @@ def run_ours(args):
     part_bytes = sum(3 * spec.shape.n_layers * spec.shape.n_kv_heads * T * 4 for T in f.Ts)
     step_s = ms / args.steps / 1e3
 
-    # e2e: the same step through the C-ABI with the inputs in pinned host memory
+    # e2e: the whole step through the C-ABI with every sender cache kept in pinned host memory.
+    # Each step copies K (and Q) to the device -- cb_score reads K twice, through tensor maps --
+    # while V stays on the host and the compaction reads only the selected V rows across the
+    # link; the send buffer and the indices come back.  Two steps are in flight, each set with its
+    # own context, device buffers and stream, so one step's copies overlap the other's kernels
+    # (a serving loop); every step still does all of its own copies.
     e2e = None
     if not args.no_e2e:
         hK = [K.cpu().pin_memory() for K, _ in inputs]
         hV = [V.cpu().pin_memory() for _, V in inputs]
         hQ = [q.cpu().pin_memory() for q in w.queries]
-        hko = torch.empty(f.k_out.shape, dtype=f.k_out.dtype).pin_memory()
-        hvo = torch.empty_like(hko).pin_memory()
-        hidx = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in f.idx]
-        h2d = sum(x.numel() * x.element_size() for x in hK + hV + hQ)
-        d2h = hko.numel() * 2 * 2 + sum(x.numel() * 4 for x in hidx)
+        state_of = {K.data_ptr(): i for i, (K, _) in enumerate(inputs)}
+        pair_state = [state_of[(K.k_pool if args.paged else K).data_ptr()] for K in f.Ks]
+        sets = []
+        for k in range(2):
+            ck = c if k == 0 else cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads,
+                                               spec.shape.head_dim, spec.m, max(spec.T), len(senders))
+            dK = [torch.empty_like(K) for K, _ in inputs]
+            dQ = [torch.empty_like(q) for q in w.queries]
+            if args.paged:
+                snd = [cb.PagedKV(dK[i], hV[i], f.Ks[j].pages, f.Ks[j].T) for j, i in enumerate(pair_state)]
+            else:
+                snd = [(dK[i], hV[i]) for i in pair_state]
+            fk = cb.Filter(ck, snd, [dQ[s_.task] for s_ in w.senders], keep, device=dev)
+            sets.append(dict(ctx=ck, dK=dK, dQ=dQ, f=fk, stream=torch.cuda.Stream(dev),
+                             hko=torch.empty(fk.k_out.shape, dtype=fk.k_out.dtype).pin_memory(),
+                             hvo=torch.empty(fk.v_out.shape, dtype=fk.v_out.dtype).pin_memory(),
+                             hidx=[torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in fk.idx]))
+        sh = spec.shape
+        v_rows = sum(b * sh.n_layers * sh.n_kv_heads * sh.head_dim * 2 for b in f.budgets)
+        h2d = sum(x.numel() * x.element_size() for x in hK + hQ) + v_rows
+        d2h = sets[0]["hko"].numel() * 2 * 2 + sum(x.numel() * 4 for x in sets[0]["hidx"])
 
-        def e2e_step():
-            for (K, V), hk, hv in zip(inputs, hK, hV):
-                K.copy_(hk, non_blocking=True)
-                V.copy_(hv, non_blocking=True)
-            for q, hq in zip(w.queries, hQ):
-                q.copy_(hq, non_blocking=True)
-            f.run(stream, wave=wave)
-            hko.copy_(f.k_out, non_blocking=True)
-            hvo.copy_(f.v_out, non_blocking=True)
-            for x, hx in zip(f.idx, hidx):
-                hx.copy_(x, non_blocking=True)
+        def e2e_step(st):
+            with torch.cuda.stream(st["stream"]):
+                for d, h in zip(st["dK"], hK):
+                    d.copy_(h, non_blocking=True)
+                for d, h in zip(st["dQ"], hQ):
+                    d.copy_(h, non_blocking=True)
+                st["f"].run(st["stream"], wave=wave)
+                st["hko"].copy_(st["f"].k_out, non_blocking=True)
+                st["hvo"].copy_(st["f"].v_out, non_blocking=True)
+                for x, hx in zip(st["f"].idx, st["hidx"]):
+                    hx.copy_(x, non_blocking=True)
 
-        n_e2e = max(2, min(args.steps, 5))
-        for _ in range(2):
-            e2e_step()
+        n_e2e = max(4, min(args.steps, 8))
+        for k in range(4):
+            e2e_step(sets[k & 1])
         torch.cuda.synchronize(dev)
         barrier(ws)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(n_e2e):
-            e2e_step()
-        e1.record(stream)
+        e0.record(sets[0]["stream"])
+        sets[1]["stream"].wait_event(e0)
+        for k in range(n_e2e):
+            e2e_step(sets[k & 1])
+        sets[0]["stream"].wait_stream(sets[1]["stream"])
+        e1.record(sets[0]["stream"])
         torch.cuda.synchronize(dev)
         barrier(ws)
+        for st in sets:
+            st["ctx"].sync_status(st["stream"])
+        # the pipelined result equals the device-resident step's
+        assert torch.equal(sets[(n_e2e - 1) & 1]["hvo"].view(torch.int16), f.v_out.cpu().view(torch.int16))
         ems = max_over_ranks(ws, e0.elapsed_time(e1))
         e2e = {"value": tokens_per_rank * ws * n_e2e / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "steps": n_e2e,
-               "ms_per_step": ems / n_e2e}
+               "d2h_bytes_per_step": d2h, "steps": n_e2e, "ms_per_step": ems / n_e2e,
+               "inputs": "K, V, Q in pinned host memory: K and Q copied each step, V read in place "
+                         "(only the selected rows cross the link)",
+               "pipeline": "two steps in flight (two contexts and streams)"}
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,

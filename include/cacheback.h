@@ -203,6 +203,10 @@ cb_status cb_select(cb_ctx *ctx, int32_t n, const float *const *scores, const in
  * (l, g) in the output; out_offset[i] + budget[i] <= out_capacity is required.
  * Indices outside [0, T_i) are skipped by the kernel and reported as CB_EDEVICE by the
  * next cb_sync_status().
+ * K_i and V_i may be device memory or pinned host memory mapped into the device (cudaHostAlloc,
+ * cudaHostRegister): the kernel then reads only the selected rows across the host link, e.g. a
+ * sender cache kept on the host whose K was copied to the device for cb_score while its V stays
+ * put.  Outputs, indices and block tables are device memory.
  * Errors: CB_EINVAL, CB_ESHAPE, CB_EBUDGET (capacity overflow).
  */
 cb_status cb_compact(cb_ctx *ctx, int32_t n, const cb_kv *senders, const int32_t *const *idx,
@@ -232,13 +236,15 @@ cb_status cb_compact_rope(cb_ctx *ctx, int32_t n, const cb_kv *senders, const in
  * selected source positions as token IDs (a table of 4-byte rows) and the latent positions as
  * continuous rows.  Both are this gather, for each sender i:
  *     out row (out_offset[i] + j) = row idx[i][j] of src[i],   j < count[i]
- *   src[i]       device table, row t (t < T[i]) at src[i] + t * src_stride bytes
+ *   src[i]       table, row t (t < T[i]) at src[i] + t * src_stride bytes: device memory, or
+ *                pinned host memory mapped into the device (only the selected rows are read)
  *   row_bytes    bytes per row, a positive multiple of 4 (src_stride, out_stride likewise, >= row_bytes)
  *   idx[i]       device int32 [count[i]] (e.g. cb_select's output or a sub-range of it)
  *   out          device buffer, row r at out + r * out_stride bytes, r < out_capacity
  * Pointers need 4-byte alignment; rows of 16-byte multiples at 16-byte aligned addresses move
- * as 16-byte pieces.  Asynchronous on `stream`; the caller owns every buffer.  Host errors: CB_EINVAL (NULL pointers, bad sizes
- * or strides, host memory), CB_ESHAPE (n < 1, T < 1), CB_EBUDGET (count < 0 or rows past
+ * as 16-byte pieces.  Asynchronous on `stream`; the caller owns every buffer.  Host errors:
+ * CB_EINVAL (NULL pointers, bad sizes or strides, unmapped host memory), CB_ESHAPE (n < 1, T < 1),
+ * CB_EBUDGET (count < 0 or rows past
  * out_capacity).  An index outside [0, T[i]) skips its row and is reported by cb_sync_status as
  * CB_EDEVICE.
  */

@@ -120,6 +120,33 @@ cb_status check_device_ptr(cb_ctx* ctx, const void* p, const char* what, int i, 
     return CB_OK;
 }
 
+// A row source the kernels may read across the host link: device memory, or pinned host memory
+// mapped into the device's address space (cudaHostAlloc / cudaHostRegister).  *dev receives the
+// address to use on the device.
+cb_status check_source_ptr(cb_ctx* ctx, const void* p, const char* what, int i, int align, const void** dev) {
+    if (!p) return fail(ctx, CB_EINVAL, "%s[%d] is NULL", what, i);
+    if (reinterpret_cast<uintptr_t>(p) % (uintptr_t)align != 0)
+        return fail(ctx, CB_EINVAL, "%s[%d] is not %d-byte aligned", what, i, align);
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ctx, CB_EINVAL, "%s[%d]: cannot query pointer", what, i);
+    }
+    if (a.type == cudaMemoryTypeHost) {
+        if (!a.devicePointer)
+            return fail(ctx, CB_EINVAL, "%s[%d] is pinned host memory not mapped into the device", what, i);
+        // the offset of p inside its allocation carries over to the device mapping
+        const uintptr_t off = reinterpret_cast<uintptr_t>(p) - reinterpret_cast<uintptr_t>(a.hostPointer);
+        *dev = static_cast<const uint8_t*>(a.devicePointer) + off;
+        if (reinterpret_cast<uintptr_t>(*dev) % (uintptr_t)align != 0)
+            return fail(ctx, CB_EINVAL, "%s[%d]: device mapping is not %d-byte aligned", what, i, align);
+        return CB_OK;
+    }
+    cb_status st = check_device_ptr(ctx, p, what, i, align);
+    if (st == CB_OK) *dev = p;
+    return st;
+}
+
 bool stride_ok(int64_t s) { return s > 0 && (s % 8) == 0; }
 
 // The optional block table of a sender (paged layout).
@@ -507,6 +534,7 @@ cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32
     cb_status st;
     if ((st = check_device_ptr(ctx, k_out, "k_out", 0))) return st;
     if ((st = check_device_ptr(ctx, v_out, "v_out", 0))) return st;
+    std::vector<const void*> kdev(n), vdev(n);
     for (int i = 0; i < n; ++i) {
         const cb_kv& s = senders[i];
         if (s.T < 1 || s.T > c.max_positions)
@@ -521,8 +549,9 @@ cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32
             return fail(ctx, CB_ESHAPE, "sender %d: too many rows for one launch", i);
         if (!stride_ok(s.s_layer) || !stride_ok(s.s_head) || !stride_ok(s.s_pos) || s.s_pos < c.head_dim)
             return fail(ctx, CB_EINVAL, "senders[%d]: strides must be positive multiples of 8 (s_pos >= d)", i);
-        if ((st = check_device_ptr(ctx, s.k, "senders.k", i))) return st;
-        if ((st = check_device_ptr(ctx, s.v, "senders.v", i))) return st;
+        // K and V rows may come from mapped pinned host memory (only the selected rows cross the link)
+        if ((st = check_source_ptr(ctx, s.k, "senders.k", i, 16, &kdev[i]))) return st;
+        if ((st = check_source_ptr(ctx, s.v, "senders.v", i, 16, &vdev[i]))) return st;
         if ((st = check_pages(ctx, s, i))) return st;
         if (budget[i] > 0 && (st = check_device_ptr(ctx, idx[i], "idx", i))) return st;
     }
@@ -543,8 +572,8 @@ cb_status compact_impl(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
             cbk::CompactSender& d = bt.s[k];
-            d.k = static_cast<const uint16_t*>(s.k);
-            d.v = static_cast<const uint16_t*>(s.v);
+            d.k = static_cast<const uint16_t*>(kdev[b0 + k]);
+            d.v = static_cast<const uint16_t*>(vdev[b0 + k]);
             d.idx = idx[b0 + k];
             d.T = s.T;
             d.ks_l = s.s_layer; d.ks_h = s.s_head; d.ks_p = s.s_pos;
@@ -635,6 +664,7 @@ cb_status cb_gather(cb_ctx* ctx, int32_t n, const void* const* src, const int64_
     if (!dg.ok) return fail(ctx, CB_ECUDA, "cannot select device %d", ctx->device);
     cb_status st;
     if ((st = check_device_ptr(ctx, out, "out", 0, 4))) return st;
+    std::vector<const void*> sdev(n);
     for (int i = 0; i < n; ++i) {
         if (T[i] < 1) return fail(ctx, CB_ESHAPE, "T[%d] = %lld < 1", i, (long long)T[i]);
         if (count[i] < 0) return fail(ctx, CB_EBUDGET, "count[%d] = %lld < 0", i, (long long)count[i]);
@@ -643,7 +673,7 @@ cb_status cb_gather(cb_ctx* ctx, int32_t n, const void* const* src, const int64_
                         (long long)out_offset[i], (long long)(out_offset[i] + count[i]), (long long)out_capacity);
         if (count[i] * (row_bytes / 4) >= ((int64_t)1 << 40))
             return fail(ctx, CB_ESHAPE, "sender %d: message too large", i);
-        if ((st = check_device_ptr(ctx, src[i], "src", i, 4))) return st;
+        if ((st = check_source_ptr(ctx, src[i], "src", i, 4, &sdev[i]))) return st;
         if (count[i] > 0 && (st = check_device_ptr(ctx, idx[i], "idx", i, 4))) return st;
     }
     cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
@@ -658,7 +688,7 @@ cb_status cb_gather(cb_ctx* ctx, int32_t n, const void* const* src, const int64_
         bt.err = ctx->err;
         for (int k = 0; k < nb; ++k) {
             cbk::GatherSender& d = bt.s[k];
-            d.src = static_cast<const uint8_t*>(src[b0 + k]);
+            d.src = static_cast<const uint8_t*>(sdev[b0 + k]);
             d.idx = idx[b0 + k];
             d.T = T[b0 + k];
             d.src_stride = src_stride;
