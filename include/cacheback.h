@@ -259,11 +259,13 @@ cb_status cb_sync_status(cb_ctx *ctx, void *stream);
 /*
  * Per-kernel timing of cb_score (tracing).  While enabled, every cb_score records CUDA events on
  * its stream between its internal kernels (no synchronisation, a few microseconds of overhead).
+ * enable: 0 off, 1 every stage, 2 only the normalised accumulation (two events around each of
+ * its launches, the least overhead).
  * cb_stage_times waits for the last recorded event and writes, into ms[0..3], the summed
  * milliseconds since the previous read of the four score kernels: row statistics (first logit
- * pass), statistics combine, normalised accumulation (second logit pass), finalize; *calls
- * receives the number of cb_score calls covered.  The sums are then reset.  Errors: CB_EINVAL
- * (timing not enabled, NULL arguments), CB_ECUDA.
+ * pass), statistics combine, normalised accumulation (second logit pass), finalize (0 for the
+ * stages not timed); *calls receives the number of cb_score calls covered.  The sums are then
+ * reset.  Errors: CB_EINVAL (timing not enabled, NULL arguments, enable outside 0..2), CB_ECUDA.
  */
 cb_status cb_enable_stage_timing(cb_ctx *ctx, int32_t enable);
 cb_status cb_stage_times(cb_ctx *ctx, float *ms, int32_t *calls);

@@ -321,8 +321,10 @@ class CacheBack:
 
     STAGES = ("row_statistics", "statistics_combine", "normalised_accumulation", "finalize")
 
-    def enable_stage_timing(self, enable: bool = True):
-        self._check(self.lib.cb_enable_stage_timing(self.h, 1 if enable else 0))
+    def enable_stage_timing(self, enable=True):
+        """True / 1: time every score kernel; 2: only the second logit pass; False / 0: off."""
+        mode = int(enable) if not isinstance(enable, bool) else (1 if enable else 0)
+        self._check(self.lib.cb_enable_stage_timing(self.h, mode))
 
     def stage_times(self):
         """(dict stage -> summed ms, number of cb_score calls) since the previous read."""

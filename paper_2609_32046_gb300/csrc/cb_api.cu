@@ -24,6 +24,7 @@ struct StageTimer {
     std::vector<std::pair<int, cudaEvent_t>> marks;
     size_t used = 0;
     int calls = 0;
+    int mode = 1;   // 1: every stage; 2: the second logit pass only (two events a launch)
     ~StageTimer() {
         for (cudaEvent_t e : pool) cudaEventDestroy(e);
     }
@@ -31,6 +32,7 @@ struct StageTimer {
 
 void stage_mark(StageTimer* t, int stage, cudaStream_t st) {
     if (!t) return;
+    if (t->mode == 2 && stage != kStageCombine && stage != kStageAccum) return;   // brackets pass 2 only
     if (t->used == t->pool.size()) {
         cudaEvent_t e;
         if (cudaEventCreate(&e) != cudaSuccess) { cudaGetLastError(); return; }
@@ -611,7 +613,9 @@ cb_status cb_compact_rope(cb_ctx* ctx, int32_t n, const cb_kv* senders, const in
 cb_status cb_enable_stage_timing(cb_ctx* ctx, int32_t enable) {
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     DeviceGuard dg(ctx->device);
+    if (enable < 0 || enable > 2) return fail(ctx, CB_EINVAL, "enable = %d not in {0, 1, 2}", enable);
     if (enable && !ctx->timer) ctx->timer = new cbk::StageTimer();
+    if (enable) ctx->timer->mode = enable;
     if (!enable && ctx->timer) {
         cudaDeviceSynchronize();
         delete ctx->timer;
@@ -634,6 +638,7 @@ cb_status cb_stage_times(cb_ctx* ctx, float* ms, int32_t* calls) {
         for (size_t i = 1; i < t->marks.size(); ++i) {
             const int stage = t->marks[i].first;
             if (stage == cbk::kStageStart) continue;
+            if (t->mode == 2 && stage != cbk::kStageAccum) continue;
             float x = 0.f;
             if (cudaEventElapsedTime(&x, t->marks[i - 1].second, t->marks[i].second) == cudaSuccess)
                 ms[stage - 1] += x;
