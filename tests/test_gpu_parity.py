@@ -227,6 +227,20 @@ def test_stage_timing_counts_calls_across_sender_batches():
     assert c.score_path() == 2
     assert calls == 3
     assert all(v > 0 for v in st.values()), st
+    # mode 2: only the second logit pass is bracketed (both sub-batches of each call)
+    c.enable_stage_timing(2)
+    c.stage_times()
+    for _ in range(3):
+        c.score(Ks, Qs, S)
+    st2, calls2 = c.stage_times()
+    assert calls2 == 3 and st2["normalised_accumulation"] > 0, st2
+    assert st2["row_statistics"] == st2["statistics_combine"] == st2["finalize"] == 0.0, st2
+    # about the same time for that kernel either way (a loose bound: timing noise)
+    assert 0.5 < st2["normalised_accumulation"] / st["normalised_accumulation"] < 2.0
+    with pytest.raises(cb.CBError) as e:
+        c.enable_stage_timing(3)
+    assert e.value.status == cb.CB_EINVAL
+    c.enable_stage_timing(False)
 
 
 def test_wave_schedule_matches_sequential():
