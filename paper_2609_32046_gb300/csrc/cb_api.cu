@@ -135,13 +135,14 @@ cb_status check_source_ptr(cb_ctx* ctx, const void* p, const char* what, int i, 
         return fail(ctx, CB_EINVAL, "%s[%d]: cannot query pointer", what, i);
     }
     if (a.type == cudaMemoryTypeHost) {
-        if (!a.devicePointer)
+        void* d = nullptr;
+        if (cudaHostGetDevicePointer(&d, const_cast<void*>(p), 0) != cudaSuccess || !d) {
+            cudaGetLastError();
             return fail(ctx, CB_EINVAL, "%s[%d] is pinned host memory not mapped into the device", what, i);
-        // the offset of p inside its allocation carries over to the device mapping
-        const uintptr_t off = reinterpret_cast<uintptr_t>(p) - reinterpret_cast<uintptr_t>(a.hostPointer);
-        *dev = static_cast<const uint8_t*>(a.devicePointer) + off;
-        if (reinterpret_cast<uintptr_t>(*dev) % (uintptr_t)align != 0)
+        }
+        if (reinterpret_cast<uintptr_t>(d) % (uintptr_t)align != 0)
             return fail(ctx, CB_EINVAL, "%s[%d]: device mapping is not %d-byte aligned", what, i, align);
+        *dev = d;
         return CB_OK;
     }
     cb_status st = check_device_ptr(ctx, p, what, i, align);
