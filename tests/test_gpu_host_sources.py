@@ -42,6 +42,21 @@ def test_compaction_reads_pinned_host_rows():
         assert_compact_exact(f, i, s.K, s.V, f.idx[i][:f.budgets[i]])
 
 
+def test_rows_inside_a_larger_pinned_allocation():
+    """A host source that starts inside its allocation (here 128 bytes in) maps to the same rows."""
+    w, c, f, dev = _setup()
+    Vs = []
+    for s in w.senders:
+        big = torch.zeros(s.V.numel() + 64, dtype=torch.bfloat16).pin_memory()
+        view = big[64:].view(s.V.shape)
+        view.copy_(s.V)
+        Vs.append(view)
+    ko, vo = torch.zeros_like(f.k_out), torch.zeros_like(f.v_out)
+    c.compact([K for K, _ in dev], Vs, f.idx, f.budgets, ko, vo, f.offsets)
+    c.sync_status()
+    assert torch.equal(vo.view(torch.int16), f.v_out.view(torch.int16))
+
+
 def test_rope_compaction_reads_pinned_host_rows():
     w, c, f, dev = _setup()
     ref_k, ref_v = torch.zeros_like(f.k_out), torch.zeros_like(f.v_out)
