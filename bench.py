@@ -296,7 +296,12 @@ def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
     t2 = time.perf_counter()
     o.compact(snd.K, snd.V, idx)
     t3 = time.perf_counter()
+    # one core: the score of a single layer (scaled like the rest)
+    t4 = time.perf_counter()
+    o.score(snd.K[:1].contiguous(), Q[:1].contiguous(), n_threads=1)
+    t5 = time.perf_counter()
     per_sender = (t1 - t0) * spec.shape.n_layers / nl + (t2 - t1) + (t3 - t2)
+    per_sender_1core = (t5 - t4) * spec.shape.n_layers + (t2 - t1) + (t3 - t2)
     total_tokens = sum(spec.T[i % len(spec.T)] for i in range(spec.n_senders))
     total_time = per_sender * spec.n_senders * (total_tokens / spec.n_senders) / snd.T
     return {
@@ -308,6 +313,9 @@ def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
                   "sender(s); fp64 C oracle, OpenMP over KV-head groups" % (
                       spec_name, nl, spec.shape.n_layers, spec.shape.n_layers / nl, spec.n_senders),
         "seconds": {"score_sample": t1 - t0, "select": t2 - t1, "compact": t3 - t2},
+        "one_core": {"value": total_tokens / (per_sender_1core * spec.n_senders * (total_tokens / spec.n_senders)
+                                               / snd.T),
+                     "sample": "one layer scored on one thread, scaled to the workload"},
     }
 
 
@@ -601,6 +609,7 @@ def run_ours(args):
                    "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential"},
         "hbm_gbs": tot_b / step_s / 1e9,
         "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
+        "hbm_frac_nominal": tot_b / step_s / 1e9 / 7900.0,   # of the 7.9 TB/s datasheet figure
         "algorithmic_bytes_per_step": tot_b,
         "step_ms": {k: v for k, v in avg.items()},
         "roofline": {
