@@ -260,7 +260,8 @@ cb_status cb_sync_status(cb_ctx *ctx, void *stream);
  * Per-kernel timing of cb_score (tracing).  While enabled, every cb_score records CUDA events on
  * its stream between its internal kernels (no synchronisation, a few microseconds of overhead).
  * enable: 0 off, 1 every stage, 2 only the normalised accumulation (two events around each of
- * its launches, the least overhead).
+ * its launches, the least overhead).  Calls captured into a CUDA graph record their events on
+ * every replay; cb_stage_times then reports the latest replay (read it once per replay).
  * cb_stage_times waits for the last recorded event and writes, into ms[0..3], the summed
  * milliseconds since the previous read of the four score kernels: row statistics (first logit
  * pass), statistics combine, normalised accumulation (second logit pass), finalize (0 for the

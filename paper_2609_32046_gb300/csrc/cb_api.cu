@@ -39,7 +39,13 @@ void stage_mark(StageTimer* t, int stage, cudaStream_t st) {
         t->pool.push_back(e);
     }
     cudaEvent_t e = t->pool[t->used++];
-    if (cudaEventRecord(e, st) != cudaSuccess) { cudaGetLastError(); return; }
+    // inside a stream capture the mark must become a graph node that records on every replay
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) cudaGetLastError();
+    const cudaError_t r = cap == cudaStreamCaptureStatusActive
+                              ? cudaEventRecordWithFlags(e, st, cudaEventRecordExternal)
+                              : cudaEventRecord(e, st);
+    if (r != cudaSuccess) { cudaGetLastError(); return; }
     t->marks.emplace_back(stage, e);   // one call may hold several sender batches: cb_score counts calls
 }
 }  // namespace cbk
