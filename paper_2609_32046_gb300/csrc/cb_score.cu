@@ -275,6 +275,41 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
     const int s = (int)(blk / nrb);
     const int row = (int)(blk % nrb) * kCombRows + (threadIdx.x & (kCombRows - 1));
     const int j = threadIdx.x / kCombRows;   // slot lane 0..3
+    const int lr = threadIdx.x & (kCombRows - 1);
+    const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
+    const int r_tok = row / G, hh = row - r_tok * G;
+    const uint16_t* qrow = sd.q + (int64_t)l * sd.qs_l + (int64_t)r_tok * sd.qs_t + (int64_t)(g * G + hh) * sd.qs_h;
+    // one logit (log2 domain) into the running offset M and sum L
+    auto merge_logit = [](float x, float& M, float& L) {
+        if (x > M) {
+            L = (M == -INFINITY ? 0.f : L * ex2(M - x)) + 1.f;
+            M = x;
+        } else {
+            L += ex2(x - M);
+        }
+    };
+    // <q_row, k> in fp32 over the head dimension (bf16 inputs)
+    auto dot_row = [&](const uint16_t* krow) {
+        float dot = 0.f;
+        for (int k = 0; k < bt.head_dim; k += 8) {
+            const uint4 a = *reinterpret_cast<const uint4*>(qrow + k);
+            const uint4 b = *reinterpret_cast<const uint4*>(krow + k);
+            const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                dot = fmaf(__uint_as_float(aw[w] << 16), __uint_as_float(bw[w] << 16), dot);
+                dot = fmaf(__uint_as_float(aw[w] & 0xFFFF0000u), __uint_as_float(bw[w] & 0xFFFF0000u), dot);
+            }
+        }
+        return dot;
+    };
+    // the query tokens' own keys: row (token r, head h) also attends to query keys 0..r (every
+    // fourth one on this slot lane); logits in the statistics' log2 domain
+    auto merge_self_keys = [&](float& M, float& L) {
+        for (int u = j; u <= r_tok; u += 4)
+            merge_logit(dot_row(sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h) *
+                            bt.scale_log2e, M, L);
+    };
     float M = -INFINITY, L = 0.f;
     if (row < R) {
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
@@ -298,36 +333,27 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
                 }
             }
         }
-        if (sd.kself) {
-            // the query tokens' own keys: row (token r, head h) also attends to query keys
-            // 0..r (every fourth one on this slot lane); logits in the statistics' log2 domain
-            const int r = row / G, hh = row - r * G;
-            const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
-            const uint16_t* qrow = sd.q + (int64_t)l * sd.qs_l + (int64_t)r * sd.qs_t + (int64_t)(g * G + hh) * sd.qs_h;
-            for (int u = j; u <= r; u += 4) {
-                const uint16_t* krow = sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h;
-                float dot = 0.f;
-                for (int k = 0; k < bt.head_dim; k += 8) {
-                    const uint4 a = *reinterpret_cast<const uint4*>(qrow + k);
-                    const uint4 b = *reinterpret_cast<const uint4*>(krow + k);
-                    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-                    for (int w = 0; w < 4; ++w) {
-                        dot = fmaf(__uint_as_float(aw[w] << 16), __uint_as_float(bw[w] << 16), dot);
-                        dot = fmaf(__uint_as_float(aw[w] & 0xFFFF0000u), __uint_as_float(bw[w] & 0xFFFF0000u), dot);
-                    }
-                }
-                const float x = dot * bt.scale_log2e;
-                if (x > M) {
-                    L = (M == -INFINITY ? 0.f : L * ex2(M - x)) + 1.f;
-                    M = x;
-                } else {
-                    L += ex2(x - M);
-                }
-            }
-        }
+        if (sd.kself) merge_self_keys(M, L);
     }
-    part[j][threadIdx.x & (kCombRows - 1)] = make_float2(M, L);
+    // A chunk partial whose sum left fp32 range makes the row's sum infinite (pass 1 of the
+    // tensor-memory path offsets each chunk by the maximum of its first 32 logits, so a logit far
+    // larger later in the chunk overflows exp2).  Such rows, rare, are recomputed here from Q and
+    // K directly: the four slot lanes take every fourth sender position.
+    __shared__ int bad[4][kCombRows];
+    part[j][lr] = make_float2(M, L);
+    bad[j][lr] = row < R && !(L <= FLT_MAX);
+    __syncthreads();
+    if (row < R && (bad[0][lr] | bad[1][lr] | bad[2][lr] | bad[3][lr])) {
+        M = -INFINITY;
+        L = 0.f;
+        const uint16_t* kbase = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
+        for (int64_t t = j; t < sd.T; t += 4) {
+            const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
+            merge_logit(ro < 0 ? 0.f : dot_row(kbase + ro) * bt.scale_log2e, M, L);   // a bad page reads as zeros
+        }
+        if (sd.kself) merge_self_keys(M, L);
+        part[j][lr] = make_float2(M, L);
+    }
     __syncthreads();
     if (j != 0 || row >= rows) return;
     float off = 0.f;

@@ -257,8 +257,10 @@ __device__ __forceinline__ void mma_k128(uint32_t d_tmem, uint32_t a_base, uint3
 }
 
 // One 32-column block of pass 1 for this lane's row: running offset m (log2 domain) and
-// sum of exp2(c z - m).  The first block sets m to its max; later blocks reuse m and are
-// redone with their own max only if their sum could leave fp32 range (rare).
+// sum of exp2(c z - m).  The first block of a chunk sets m to its max; later blocks reuse m
+// without a check (a per-block test and redo cost 11% of this kernel).  Values up to 2^127 above
+// the first block are exact; a logit so far above it that exp2 or the sum overflows leaves an
+// infinite sum, and the combine kernel recomputes that row's statistics from Q and K.
 __device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c, uint64_t cc, float& m, float& sum) {
     if (nvalid < 32) {
 #pragma unroll
@@ -266,7 +268,7 @@ __device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c,
     }
     if (m == -INFINITY) m = max_tree1(v) * c;
     if (m == -INFINITY) return;
-    uint64_t nm = pack2(-m, -m);
+    const uint64_t nm = pack2(-m, -m);
     float acc[4] = {0.f, 0.f, 0.f, 0.f};   // exp2 results are summed as scalars (no pair packing)
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
@@ -275,23 +277,7 @@ __device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c,
         acc[(2 * q) & 3] += ex2(a0);
         acc[(2 * q + 1) & 3] += ex2(a1);
     }
-    float blk = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-    if (!(blk <= 0x1p64f)) {
-        const float mn = fmaxf(m, max_tree1(v) * c);
-        nm = pack2(-mn, -mn);
-        acc[0] = acc[1] = acc[2] = acc[3] = 0.f;
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-            float a0, a1;
-            unpack2(ffma2(pack2(v[2 * q], v[2 * q + 1]), cc, nm), a0, a1);
-            acc[(2 * q) & 3] += ex2(a0);
-            acc[(2 * q + 1) & 3] += ex2(a1);
-        }
-        blk = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-        sum *= ex2(m - mn);
-        m = mn;
-    }
-    sum += blk;
+    sum += (acc[0] + acc[1]) + (acc[2] + acc[3]);
 }
 
 // ===========================================================================

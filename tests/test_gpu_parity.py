@@ -261,3 +261,23 @@ def test_wave_schedule_matches_sequential():
     assert torch.equal(ref.k_out.view(torch.int16), got.k_out.view(torch.int16))
     assert torch.equal(ref.v_out.view(torch.int16), got.v_out.view(torch.int16))
 
+
+
+@pytest.mark.parametrize("kernel", [1, 2], ids=["mma_sync", "tcgen05"])
+@pytest.mark.parametrize("scale", [70.0, 150.0], ids=["large_finite", "overflowing"])
+def test_extreme_logit_rows(kernel, scale):
+    """One query row meets keys far above the rest of its chunk: c*z - m about 100 log2 units stays
+    in fp32 range on the fast path, about 210 overflows pass 1's exp2 and the combine kernel
+    recomputes that row's statistics from Q and K.  Scores must still match the oracle."""
+    w = synth.custom_workload(synth.Shape(2, 8, 2, 128), [700], 8, seed=77, n_planted_spans=2)
+    s = w.senders[0]
+    K, V, Q = s.K.clone(), s.V, w.queries[0]
+    l, r, h = 1, 3, 5
+    g = h // 4
+    q = Q[l, r, h].float()
+    K[l, g, 300:304] = (q / q.norm() * scale).to(torch.bfloat16)
+    c = make_cb(w.spec.shape, 700, 8, 1, score_kernel=kernel)
+    f = cb.Filter(c, [(K.cuda(), V.cuda())], [Q.cuda()], 0.25).run()
+    c.sync_status()
+    assert c.score_path() == kernel
+    check_sender(f, 0, K, V, Q)
