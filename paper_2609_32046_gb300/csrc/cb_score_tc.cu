@@ -418,7 +418,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                     for (int half32 = 0; half32 < 2; ++half32) {
                         float v[32];
                         tmem_ld32(ta + 32 * half32, v);
-                        tmem_wait_ld();
+                        tmem_wait_ld(v);
                         if (half32 == 1) {
                             tc_fence_before();
                             __syncwarp();
@@ -726,7 +726,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     for (int col = 0; col < (G == 4 ? 0 : ncol); col += 32) {
                         float v[32];
                         tmem_ld32(ta + col, v);
-                        tmem_wait_ld();
+                        tmem_wait_ld(v);
                         accum_block<G, PH, P2>(v, cc, valid, all_valid, bt.p, bt.p_inf, nacc2, bsum2);
                     }
                     tc_fence_before();
