@@ -257,17 +257,19 @@ __device__ __forceinline__ void mma_k128(uint32_t d_tmem, uint32_t a_base, uint3
 }
 
 // One 32-column block of pass 1 for this lane's row: running offset m (log2 domain) and
-// sum of exp2(c z - m).  The first block of a chunk sets m to its max; later blocks reuse m
-// without a check (a per-block test and redo cost 11% of this kernel).  Values up to 2^127 above
+// sum of exp2(c z - m).  The first block of a chunk (known from the loop indices: testing m
+// instead cost 2%) sets m to its max, or to -FLT_MAX when it holds no position, in which case
+// neither does the rest of the chunk; later blocks reuse m without a check (a per-block test
+// and redo cost 11% of this kernel).  Values up to 2^127 above
 // the first block are exact; a logit so far above it that exp2 or the sum overflows leaves an
 // infinite sum, and the combine kernel recomputes that row's statistics from Q and K.
-__device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c, uint64_t cc, float& m, float& sum) {
+__device__ __forceinline__ void stats_block(float (&v)[32], int nvalid, float c, uint64_t cc, float& m, float& sum,
+                                            bool first) {
     if (nvalid < 32) {
 #pragma unroll
         for (int q = 0; q < 32; ++q) v[q] = q < nvalid ? v[q] : -INFINITY;
     }
-    if (m == -INFINITY) m = max_tree1(v) * c;
-    if (m == -INFINITY) return;
+    if (first) m = fmaxf(max_tree1(v) * c, -FLT_MAX);
     const uint64_t nm = pack2(-m, -m);
     float acc[4] = {0.f, 0.f, 0.f, 0.f};   // exp2 results are summed as scalars (no pair packing)
 #pragma unroll
@@ -424,7 +426,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
                             __syncwarp();
                             if (lane == 0) mbar_arrive(&ctl->t_empty[buf]);   // registers hold the rest
                         }
-                        stats_block(v, nvalid - 32 * half32, c, cc, m, sum);
+                        stats_block(v, nvalid - 32 * half32, c, cc, m, sum, tile == grp && half32 == 0);
                     }
                     M[h] = m;
                     S[h] = sum;
@@ -432,7 +434,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
             }
             if (!ok) break;
             // this warp's partial statistics for the chunk: slot 4 c + 2 grp + hf (rows of
-            // tiles it saw none of stay (-inf, 0)); the combine kernel merges all slots
+            // tiles it saw none of stay (-inf, 0), rows of positions past T (-FLT_MAX, 0), both
+            // of which add nothing); the combine kernel merges all slots
             float2* dst = sd.stats + ((int64_t)un.s * sd.n_chunk1 + 4 * un.c + 2 * grp + hf) * sd.R;
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
