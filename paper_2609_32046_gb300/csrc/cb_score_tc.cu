@@ -84,7 +84,8 @@ struct TcBatch {
 
 struct Ctl {
     uint64_t k_full[kMaxStages], k_empty[kMaxStages];
-    uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns; group g owns 2g and 2g + 1
+    uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns (pass 1: group g owns 2g and 2g + 1;
+                                      // pass 2: buffer 2g + h is column half h of group g)
     uint64_t q_full, q_empty, drain, o_full;
     uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]
     uint32_t tmem_base;
@@ -201,14 +202,16 @@ __device__ __forceinline__ Smem carve(uint8_t* raw, const TcBatch& bt) {
     return sm;
 }
 
-__device__ __forceinline__ void init_ctl(Ctl* ctl, int stages) {
+// `releasers`: warps that arrive on a TMEM buffer's empty barrier (pass 1: the eight warps of a
+// group; pass 2: the four warps of one column half).
+__device__ __forceinline__ void init_ctl(Ctl* ctl, int stages, int releasers) {
     for (int k = 0; k < stages; ++k) {
         mbar_init(&ctl->k_full[k], 1);
         mbar_init(&ctl->k_empty[k], 1);
     }
     for (int b = 0; b < 4; ++b) {
         mbar_init(&ctl->t_full[b], 1);
-        mbar_init(&ctl->t_empty[b], 8);   // the eight warps of the group that owns the tile
+        mbar_init(&ctl->t_empty[b], releasers);
     }
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
@@ -294,7 +297,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     const Smem sm = carve(smem_raw, bt);
     Ctl* ctl = sm.ctl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) init_ctl(ctl, bt.stages);
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 8);
     if (warp == 1) {
         tmem_alloc(&ctl->tmem_base, kTmemCols);
         tmem_relinquish();
@@ -479,6 +482,8 @@ __device__ __forceinline__ float pow_p(float x, float p) {
 
 // One 32-column block of pass 2 for this lane's position: a / G = exp2(c z - offset) per
 // column, b = sum over the G heads of each token, then Pool over positions and the sums.
+// Tokens 2i and 2i + 1 share one packed f32x2 add or fma: lane 0 of each pair is the chain of
+// even tokens and lane 1 that of odd tokens, the same order of additions as two scalar chains.
 template <int G, int PH, bool P2>
 __device__ __forceinline__ void accum_block(const float (&v)[32], uint64_t cc, bool valid, bool all_valid, float p,
                                             bool p_inf, float (&nacc)[2], float (&bsum)[2]) {
@@ -493,32 +498,46 @@ __device__ __forceinline__ void accum_block(const float (&v)[32], uint64_t cc, b
         e[4 * q + 2] = ex2(a2);
         e[4 * q + 3] = ex2(a3);
     }
-    constexpr int NT = 32 / G;   // tokens in these 32 columns
-    float b[NT];
+    constexpr int NP = 16 / G;   // token pairs in these 32 columns
+    uint64_t b[NP];
 #pragma unroll
-    for (int k = 0; k < NT; ++k) {
-        if (G == 1) b[k] = e[k];
-        if (G == 2) b[k] = e[2 * k] + e[2 * k + 1];
-        if (G == 4) b[k] = (e[4 * k] + e[4 * k + 1]) + (e[4 * k + 2] + e[4 * k + 3]);
+    for (int i = 0; i < NP; ++i) {
+        if (G == 1) b[i] = pack2(e[2 * i], e[2 * i + 1]);
+        if (G == 2) b[i] = fadd2(pack2(e[4 * i], e[4 * i + 2]), pack2(e[4 * i + 1], e[4 * i + 3]));
+        if (G == 4)
+            b[i] = fadd2(fadd2(pack2(e[8 * i], e[8 * i + 4]), pack2(e[8 * i + 1], e[8 * i + 5])),
+                         fadd2(pack2(e[8 * i + 2], e[8 * i + 6]), pack2(e[8 * i + 3], e[8 * i + 7])));
     }
     if (!all_valid) {
 #pragma unroll
-        for (int k = 0; k < NT; ++k) b[k] = valid ? b[k] : 0.f;
+        for (int i = 0; i < NP; ++i) b[i] = valid ? b[i] : 0ull;
     }
+    uint64_t bs = pack2(bsum[0], bsum[1]), na = pack2(nacc[0], nacc[1]);
 #pragma unroll
-    for (int k = 0; k < NT; ++k) {
-        const float pk = lane_pool<PH>(b[k]);
-        bsum[k & 1] += b[k];
-        if (P2) nacc[k & 1] = fmaf(pk, pk, nacc[k & 1]);
-        else if (p_inf) nacc[k & 1] = fmaxf(nacc[k & 1], pk);   // p = infinity: largest pooled value
-        else nacc[k & 1] += pow_p<false>(pk, p);
+    for (int i = 0; i < NP; ++i) {
+        float b0, b1;
+        unpack2(b[i], b0, b1);
+        const float p0 = lane_pool<PH>(b0), p1 = lane_pool<PH>(b1);
+        bs = fadd2(bs, b[i]);
+        if (P2) {
+            const uint64_t pp = pack2(p0, p1);
+            na = ffma2(pp, pp, na);
+        } else if (p_inf) {   // p = infinity: largest pooled value
+            nacc[0] = fmaxf(nacc[0], p0);
+            nacc[1] = fmaxf(nacc[1], p1);
+        } else {
+            nacc[0] += pow_p<false>(p0, p);
+            nacc[1] += pow_p<false>(p1, p);
+        }
     }
+    unpack2(bs, bsum[0], bsum[1]);
+    if (P2) unpack2(na, nacc[0], nacc[1]);
 }
 
-// Pass 2, G = 4: head sums b of the four tokens in 16 columns (exp2(c z - offset) summed
-// over each token's four heads).
-__device__ __forceinline__ void head_sums16(const float (&v)[16], uint64_t cc, float& b0, float& b1, float& b2,
-                                            float& b3) {
+// Pass 2, G = 4: head sums of the four tokens in 16 columns (exp2(c z - offset) summed over
+// each token's four heads) as the pairs (b0, b1) and (b2, b3); the packed adds keep each
+// token's order (e0 + e1) + (e2 + e3).
+__device__ __forceinline__ void head_sums16(const float (&v)[16], uint64_t cc, uint64_t& b01, uint64_t& b23) {
     float e[16];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -530,10 +549,8 @@ __device__ __forceinline__ void head_sums16(const float (&v)[16], uint64_t cc, f
         e[4 * q + 2] = ex2(a2);
         e[4 * q + 3] = ex2(a3);
     }
-    b0 = (e[0] + e[1]) + (e[2] + e[3]);
-    b1 = (e[4] + e[5]) + (e[6] + e[7]);
-    b2 = (e[8] + e[9]) + (e[10] + e[11]);
-    b3 = (e[12] + e[13]) + (e[14] + e[15]);
+    b01 = fadd2(fadd2(pack2(e[0], e[4]), pack2(e[1], e[5])), fadd2(pack2(e[2], e[6]), pack2(e[3], e[7])));
+    b23 = fadd2(fadd2(pack2(e[8], e[12]), pack2(e[9], e[13])), fadd2(pack2(e[10], e[14]), pack2(e[11], e[15])));
 }
 
 // Epilogue: each warp owns 32 TMEM lanes = positions t0 + 26 w - 3 + lane (w = lane quarter);
@@ -545,7 +562,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
     const Smem sm = carve(smem_raw, bt);
     Ctl* ctl = sm.ctl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) init_ctl(ctl, bt.stages);
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 4);
     if (warp == 1) {
         tmem_alloc(&ctl->tmem_base, kTmemCols);
         tmem_relinquish();
@@ -598,8 +615,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         }
     } else if (warp == 1) {
         if (elect_one()) {
-            int64_t qn = 0, jg0 = 0, jg1 = 0;   // Q loads consumed; items issued per epilogue group
-            int st = 0;                          // ring slot of the next K tile and its phase parity
+            int64_t qn = 0;              // Q loads consumed
+            uint32_t jpar = 0;           // bit b: parity of the items issued into TMEM buffer b
+            int st = 0;                  // ring slot of the next K tile and its phase parity
             uint32_t ph = 0;
             int prev = -1;
             bool ok = wait_bar(&ctl->o_full, 0, ctl, bt.err, 15);
@@ -620,21 +638,38 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                 if (!(ok = wait_bar(&ctl->k_full[st], ph, ctl, bt.err, 11))) break;
                 tc_fence_after();
                 const uint32_t kaddr = smem_u32(sm.k + (size_t)st * kTileBytes);
-                const int nch = (sd.R_pad + 255) / 256;
                 const int grp = (int)((u - ub) & 1);   // epilogue group that owns this tile
-                for (int c = 0; c < nch; ++c) {
-                    // group g owns the 256 columns of buffers 2g and 2g + 1 (barriers of buffer 2g)
-                    const int64_t j = grp ? jg1++ : jg0++;
-                    if (!(ok = wait_bar(&ctl->t_empty[2 * grp], (uint32_t)((j & 1) ^ 1), ctl, bt.err, 12))) break;
+                if (sd.R_pad == 256) {
+                    // both halves in one 256-column MMA (faster when the tile has no other rows);
+                    // it waits for both halves' buffers and completes both
+                    const uint32_t jp = (jpar >> (2 * grp)) & 3u;
+                    jpar ^= 3u << (2 * grp);
+                    if (!(ok = wait_bar(&ctl->t_empty[2 * grp], (jp & 1u) ^ 1u, ctl, bt.err, 12))) break;
+                    if (!(ok = wait_bar(&ctl->t_empty[2 * grp + 1], (jp >> 1) ^ 1u, ctl, bt.err, 12))) break;
                     tc_fence_after();
-                    const int ncol = min(256, sd.R_pad - 256 * c);
-                    mma_k128(tmem + grp * 256, kaddr, kTileBytes / 2, smem_u32(sm.q) + c * 256 * 128,
-                             (uint32_t)bt.rpad_max * 128, idesc_bf16_f32(128, ncol));
+                    mma_k128(tmem + grp * 256, kaddr, kTileBytes / 2, smem_u32(sm.q), (uint32_t)bt.rpad_max * 128,
+                             idesc_bf16_f32(128, 256));
                     // one more K-step: ones (positions) x offset terms (rows) adds -offset / scale to
                     // every logit, so the epilogue needs only exp2(scale * D)
-                    umma_bf16(tmem + grp * 256, ones_desc, ext_desc + (uint64_t)((c * 256 * 32) >> 4),
-                              idesc_bf16_f32(128, ncol), 1u);
+                    umma_bf16(tmem + grp * 256, ones_desc, ext_desc, idesc_bf16_f32(128, 256), 1u);
                     umma_commit(&ctl->t_full[2 * grp]);
+                    umma_commit(&ctl->t_full[2 * grp + 1]);
+                } else {
+                    // one 128-column MMA per column half, each into its own buffer, so that each
+                    // half's warps start as soon as their columns are done and release them on
+                    // their own (the next chunk waits for one half, not for the whole group)
+                    for (int r0 = 0; r0 < sd.R_pad && ok; r0 += 128) {
+                        const int b = 2 * grp + ((r0 >> 7) & 1);
+                        const uint32_t jp = (jpar >> b) & 1u;
+                        jpar ^= 1u << b;
+                        if (!(ok = wait_bar(&ctl->t_empty[b], jp ^ 1u, ctl, bt.err, 12))) break;
+                        tc_fence_after();
+                        mma_k128(tmem + b * 128, kaddr, kTileBytes / 2, smem_u32(sm.q) + r0 * 128,
+                                 (uint32_t)bt.rpad_max * 128, idesc_bf16_f32(128, 128));
+                        umma_bf16(tmem + b * 128, ones_desc, ext_desc + (uint64_t)((r0 * 32) >> 4),
+                                  idesc_bf16_f32(128, 128), 1u);
+                        umma_commit(&ctl->t_full[b]);
+                    }
                 }
                 umma_commit(&ctl->k_empty[st]);
                 if (++st == stages) { st = 0; ph ^= 1u; }
@@ -650,7 +685,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
         float2* xch = reinterpret_cast<float2*>(sm.epi);   // [parity][grp][sp][32]
         const float c = bt.sl2e;
         const uint64_t cc = pack2(c, c);
-        int64_t j = 0, gt = 0;                   // chunks and tiles of this group so far
+        int64_t j = 0, gt = 0;                   // chunks of this warp's buffer and tiles of this group so far
         int prev = -1;
         bool ok = true;
         // per-sender values live in registers and are refreshed when the group s changes
@@ -692,37 +727,59 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const bool all_valid = __all_sync(0xffffffffu, valid);
             float nacc2[2] = {0.f, 0.f}, bsum2[2] = {0.f, 0.f};   // token partial sums (two chains)
             for (int ci = 0; ci < nch && ok; ++ci) {
-                if (!(ok = wait_bar(&ctl->t_full[2 * grp], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
+                // this half's columns (R_pad is a multiple of 128: 0 or 128); a half with none has
+                // no MMA and nothing to wait for
+                const int ncol = min(128, min(256, R_pad - 256 * ci) - hf * 128);
+                if (ncol <= 0) continue;
+                if (!(ok = wait_bar(&ctl->t_full[2 * grp + hf], (uint32_t)(j & 1), ctl, bt.err, 13))) break;
                 ++j;
                 tc_fence_after();
-                const int ncol = min(128, min(256, R_pad - 256 * ci) - hf * 128);   // this half's columns
                 const uint32_t ta = tmem + lane_addr + grp * 256 + hf * 128;
-                if (G == 4 && ncol > 0) {   // R_pad is a multiple of 128: ncol is 0 or 128
+                if (G == 4) {
                     // head sums of the warp's 32 tokens first, then the buffer goes back to the MMA
-                    // while Pool and the token sums run from registers
-                    float b[32];
+                    // while Pool and the token sums run from registers; each 16-column load is
+                    // issued before the head sums of the one before it
+                    uint64_t b[16];   // (token 2i, token 2i + 1)
+                    {
+                        float va[16], vb[16];
+                        tmem_ld16(ta, va);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        float v[16];
-                        tmem_ld16(ta + 16 * k, v);
-                        tmem_wait_ld(v);
-                        head_sums16(v, cc, b[4 * k], b[4 * k + 1], b[4 * k + 2], b[4 * k + 3]);
+                        for (int k = 0; k < 8; k += 2) {
+                            tmem_wait_ld(va);
+                            tmem_ld16(ta + 16 * (k + 1), vb);
+                            head_sums16(va, cc, b[2 * k], b[2 * k + 1]);
+                            tmem_wait_ld(vb);
+                            if (k + 2 < 8) tmem_ld16(ta + 16 * (k + 2), va);
+                            head_sums16(vb, cc, b[2 * k + 2], b[2 * k + 3]);
+                        }
                     }
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
+                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp + hf]);
                     if (!all_valid) {
 #pragma unroll
-                        for (int k = 0; k < 32; ++k) b[k] = valid ? b[k] : 0.f;
+                        for (int i = 0; i < 16; ++i) b[i] = valid ? b[i] : 0ull;
                     }
+                    uint64_t bs = pack2(bsum2[0], bsum2[1]), na = pack2(nacc2[0], nacc2[1]);
 #pragma unroll
-                    for (int k = 0; k < 32; ++k) {
-                        const float pk = lane_pool<PH>(b[k]);
-                        bsum2[k & 1] += b[k];
-                        if (P2) nacc2[k & 1] = fmaf(pk, pk, nacc2[k & 1]);
-                        else if (bt.p_inf) nacc2[k & 1] = fmaxf(nacc2[k & 1], pk);
-                        else nacc2[k & 1] += pow_p<false>(pk, bt.p);
+                    for (int i = 0; i < 16; ++i) {
+                        float b0, b1;
+                        unpack2(b[i], b0, b1);
+                        const float p0 = lane_pool<PH>(b0), p1 = lane_pool<PH>(b1);
+                        bs = fadd2(bs, b[i]);
+                        if (P2) {
+                            const uint64_t pp = pack2(p0, p1);
+                            na = ffma2(pp, pp, na);
+                        } else if (bt.p_inf) {
+                            nacc2[0] = fmaxf(nacc2[0], p0);
+                            nacc2[1] = fmaxf(nacc2[1], p1);
+                        } else {
+                            nacc2[0] += pow_p<false>(p0, bt.p);
+                            nacc2[1] += pow_p<false>(p1, bt.p);
+                        }
                     }
+                    unpack2(bs, bsum2[0], bsum2[1]);
+                    if (P2) unpack2(na, nacc2[0], nacc2[1]);
                 } else {
                     // 32-column steps; sixteen epilogue warps hide the TMEM load latency
 #pragma unroll 1
@@ -734,7 +791,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
                     }
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp]);
+                    if (lane == 0) mbar_arrive(&ctl->t_empty[2 * grp + hf]);
                 }
             }
             if (!ok) break;
