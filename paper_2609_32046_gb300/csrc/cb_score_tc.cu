@@ -87,10 +87,12 @@ struct Ctl {
     uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns (pass 1: group g owns 2g and 2g + 1;
                                       // pass 2: buffer 2g + h is column half h of group g)
     uint64_t q_full, q_empty, drain, o_full;
-    uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]
+    uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]: written
+    uint64_t xe[2][2][4];   //   and read (half 1 reuses a slot only after half 0 has read it)
     uint32_t tmem_base;
     int abort;
 };
+static_assert(sizeof(Ctl) <= 512, "the epilogue exchange area starts 512 bytes after Ctl");
 
 __device__ __forceinline__ uint64_t now_ns() {
     uint64_t t;
@@ -217,7 +219,10 @@ __device__ __forceinline__ void init_ctl(Ctl* ctl, int stages, int releasers) {
     mbar_init(&ctl->q_empty, 1);
     mbar_init(&ctl->drain, 1);
     mbar_init(&ctl->o_full, 1);
-    for (int k = 0; k < 16; ++k) mbar_init(&ctl->xb[k >> 3][(k >> 2) & 1][k & 3], 1);
+    for (int k = 0; k < 16; ++k) {
+        mbar_init(&ctl->xb[k >> 3][(k >> 2) & 1][k & 3], 1);
+        mbar_init(&ctl->xe[k >> 3][(k >> 2) & 1][k & 3], 1);
+    }
     ctl->abort = 0;
     fence_barrier_init();
 }
@@ -803,13 +808,18 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const int tp = (int)(gt & 1);
             float2* xs = xch + ((tp * 2 + grp) * 4 + sp) * 32;
             uint64_t* xb = &ctl->xb[tp][grp][sp];
+            uint64_t* xe = &ctl->xe[tp][grp][sp];
             if (hf == 1) {
+                // the slot was last used two tiles ago: wait until half 0 has read it
+                if (!(ok = wait_bar(xe, (uint32_t)(((gt >> 1) & 1) ^ 1), ctl, bt.err, 7))) break;
                 xs[lane] = make_float2(nacc, bsum);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(xb);
             } else {
                 if (!(ok = wait_bar(xb, (uint32_t)((gt >> 1) & 1), ctl, bt.err, 14))) break;
                 const float2 o = xs[lane];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(xe);
                 nacc = p_inf ? fmaxf(nacc, o.x) : nacc + o.x;
                 bsum += o.y;
                 const float pb = lane_pool<PH>(bsum * inv_m);
