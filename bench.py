@@ -347,7 +347,10 @@ def run_reference(args):
     out = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": per_step_s * 1e3, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": args.workload, "keep": spec.keeps[0], "senders": spec.n_senders},
+           "config": {"workload": args.workload, "senders": spec.n_senders, "T": list(spec.T[:3]), "m": spec.m,
+                      "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
+                      "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": spec.keeps[0],
+                      "layout": "strided [nL][Hkv][T][d]", "parallelism": "single"},
            "cpu_baseline": cpu,
            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))

@@ -63,3 +63,11 @@ def test_reference_arm_under_torchrun_prints_one_line_from_rank_0():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+    # the same workload keys as the GPU arm's config
+    import synth
+    spec = synth.SPECS["tiny"]
+    sh = spec.shape
+    want = {"workload": "tiny", "senders": spec.n_senders, "T": list(spec.T[:3]), "m": spec.m,
+            "n_layers": sh.n_layers, "q_heads": sh.n_q_heads, "kv_heads": sh.n_kv_heads, "head_dim": sh.head_dim,
+            "keep": spec.keeps[0]}
+    assert {k: d["config"][k] for k in want} == want
