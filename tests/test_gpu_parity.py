@@ -31,6 +31,8 @@ CASES = [
     ("width8_spans_p1_5", (1, 8, 4, 128), [611], 9, 0.35, dict(span_width=8, p=1.5, alpha=4.0)),
     ("fan_in_ragged", (2, 16, 4, 128), [300, 513, 129], 33, 0.25, {}),
     ("m128_two_chunks", (2, 32, 8, 128), [900], 128, 0.25, {}),
+    # 384 rows with G = 4: the last 256-row chunk has only its first column half
+    ("g4_m96_three_halves", (2, 32, 8, 128), [1100], 96, 0.25, {}),
     ("g2_m200", (1, 8, 4, 128), [555], 200, 0.25, {}),
     ("g1_m300", (1, 2, 2, 128), [400], 300, 0.5, {}),
     ("pool3", (1, 8, 2, 128), [500], 40, 0.3, dict(pool_width=3)),
@@ -44,6 +46,7 @@ CASES = [
     ("p_inf_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(p=float("inf"))),
     ("p_inf_g2_pool5", (2, 8, 4, 128), [611], 20, 0.3, dict(p=float("inf"), pool_width=5, alpha=3.0)),
     ("p_inf_d64", (2, 8, 2, 64), [600], 12, 0.2, dict(p=float("inf"))),
+    ("p_inf_m128_four_halves", (1, 32, 8, 128), [700], 128, 0.3, dict(p=float("inf"))),
     # the query tokens' own keys join the softmax causally
     ("self_keys_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(self_keys=True)),
     ("self_keys_g2_d64", (2, 8, 4, 64), [333], 17, 0.3, dict(self_keys=True)),
