@@ -47,7 +47,7 @@ typedef enum {
     CB_EBUDGET = 3,  /* budget below the forced positions, above T, or beyond the output capacity */
     CB_ENOMEM = 4,   /* device allocation failed */
     CB_ECUDA = 5,    /* a CUDA runtime call or a kernel launch failed */
-    CB_ETIMEOUT = 6, /* reserved: a bounded device wait gave up */
+    CB_ETIMEOUT = 6, /* a bounded device wait gave up (see cb_set_wait_limit, cb_sync_status) */
     CB_EDEVICE = 7   /* a kernel's own bounds check rejected an input (see cb_sync_status) */
 } cb_status;
 
@@ -271,6 +271,23 @@ cb_status cb_sync_status(cb_ctx *ctx, void *stream);
 cb_status cb_enable_stage_timing(cb_ctx *ctx, int32_t enable);
 cb_status cb_stage_times(cb_ctx *ctx, float *ms, int32_t *calls);
 
+/*
+ * Bounded device waits (failure detection; the paper has no counterpart: this is a runtime
+ * control).  Every mbarrier wait of the tcgen05 score passes gives up after limit_ns
+ * nanoseconds (default 1 s): the kernel then records which wait gave up, sets an abort flag
+ * that every role of its CTA sees, waits (bounded) for its own copies and MMAs in flight,
+ * frees its tensor memory and returns, so the context stays usable; the next cb_sync_status
+ * reports CB_ETIMEOUT and that call's scores are invalid.
+ *   limit_ns          0 restores the default; otherwise 1e3 .. 6e10
+ *   stall_next_score  1: the next cb_score that runs the tcgen05 passes makes one wait of its
+ *                     first row-statistics launch (CTA 0's MMA issuer) on a barrier nothing
+ *                     arrives on, so that wait runs out after limit_ns and the path above is
+ *                     taken; cleared by that call.  For tests of failure detection; it faults
+ *                     and hangs nothing.  The mma.sync passes have no waits and ignore it.
+ * Errors: CB_EINVAL (NULL ctx, values out of range).  Host-only; affects later calls.
+ */
+cb_status cb_set_wait_limit(cb_ctx *ctx, int64_t limit_ns, int32_t stall_next_score);
+
 /* Free the context's scratch (after synchronising its device).  NULL is ignored. */
 void cb_destroy(cb_ctx *ctx);
 
@@ -296,10 +313,13 @@ int32_t cb_score_path(const cb_ctx *ctx);
  * and takes the selection parameters directly instead of from a context.
  *
  * Scratch: a fixed array of 65536 span slots (256 KiB) compiled into the library, held by
- * every GPU that loads the library until the process exits.  One call may use at most
- * 65536 slots in total, sum_i ceil(T[i] / span_width); larger calls return CB_ESHAPE
- * with nothing enqueued.  The call allocates nothing: no cudaMalloc, cudaFree or
- * allocating library routine.
+ * every GPU that loads the library until the process exits.  The selection kernel keeps the
+ * span means of a sender with at most 8192 spans in shared memory; only senders with more
+ * spans (ceil(T[i] / span_width) > 8192, e.g. T above 131072 at width 16) take slots in the
+ * array.  Senders are launched in groups of 64, each group placing its large senders from slot
+ * 0, so a call is limited to 65536 such slots per group of 64 consecutive senders; a larger
+ * call returns CB_ESHAPE with nothing enqueued.  The call allocates nothing: no cudaMalloc,
+ * cudaFree or allocating library routine.
  *
  * Set-up: the first call on each device looks up the array's device address (with that
  * device current) and caches it; make that first call before any stream capture.
@@ -308,11 +328,20 @@ int32_t cb_score_path(const cb_ctx *ctx);
  * contents in it (the kernel rewrites every slot it reads, and the call clears its status
  * word).  Calls whose kernels may overlap on the GPU race on the array: order them on one
  * stream or synchronise between them.  Arguments are as for cb_select; the current CUDA
- * device is used; errors are described by cb_last_error(NULL).
+ * device is used; host-side errors are returned at once and described by cb_last_error(NULL);
+ * the kernel's own consistency check is read back by cb_select_noalloc_status.
  */
 cb_status cb_select_noalloc(int32_t n, const float *const *scores, const int64_t *T,
                             const int64_t *budget, int32_t *const *idx, int32_t n_sink,
                             int32_t n_latent, int32_t span_width, void *stream);
+
+/* Status of the allocation-free selection (no context, no allocation): waits for `stream`,
+ * reads the status word that cb_select_noalloc's kernel keeps in the library's fixed array on
+ * the current device, clears it, and returns CB_EDEVICE (text in cb_last_error(NULL)) when the
+ * kernel's own check found a selected count different from the budget, CB_ECUDA when the
+ * stream reported an error, else CB_OK.  It covers every cb_select_noalloc call on this device
+ * since the last read.  Blocks the host. */
+cb_status cb_select_noalloc_status(void *stream);
 
 #ifdef __cplusplus
 }

@@ -13,12 +13,12 @@ from __future__ import annotations
 
 from typing import List, Optional, Sequence
 
-from .binding import (CB_EBUDGET, CB_ECUDA, CB_EDEVICE, CB_EINVAL, CB_ENOMEM, CB_ESHAPE, CB_OK, EXPORTED,
+from .binding import (CB_EBUDGET, CB_ECUDA, CB_EDEVICE, CB_EINVAL, CB_ENOMEM, CB_ESHAPE, CB_ETIMEOUT, CB_OK, EXPORTED,
                       LIB_PATH, CacheBack, CBError, PagedKV, budget, chain_budget, load_library)
 
 __all__ = ["CacheBack", "CBError", "PagedKV", "budget", "chain_budget", "load_library", "LIB_PATH", "EXPORTED",
            "Filter", "Chain",
-           "CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_EDEVICE"]
+           "CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "CB_ECUDA", "CB_ETIMEOUT", "CB_EDEVICE"]
 
 
 class Filter:

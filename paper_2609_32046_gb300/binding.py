@@ -21,8 +21,8 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 # Every entry point include/cacheback.h declares (checked by the tests).
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
             "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
-            "cb_gather", "cb_chain_budget", "cb_compact_rope",
-            "cb_enable_stage_timing", "cb_stage_times"]
+            "cb_select_noalloc_status", "cb_gather", "cb_chain_budget", "cb_compact_rope",
+            "cb_enable_stage_timing", "cb_stage_times", "cb_set_wait_limit"]
 
 
 class CBError(RuntimeError):
@@ -102,6 +102,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_score_path.restype = ctypes.c_int32
     lib.cb_select_noalloc.argtypes = [ctypes.c_int32, P, P, P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
     lib.cb_select_noalloc.restype = ctypes.c_int
+    lib.cb_set_wait_limit.argtypes = [P, ctypes.c_int64, ctypes.c_int32]
+    lib.cb_set_wait_limit.restype = ctypes.c_int
+    lib.cb_select_noalloc_status.argtypes = [P]
+    lib.cb_select_noalloc_status.restype = ctypes.c_int
     lib.cb_enable_stage_timing.argtypes = [P, ctypes.c_int32]
     lib.cb_enable_stage_timing.restype = ctypes.c_int
     lib.cb_stage_times.argtypes = [P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int32)]
@@ -136,6 +140,15 @@ def select_noalloc(scores: Sequence, Ts: Sequence[int], budgets: Sequence[int], 
                                _ptr_array([int(b) for b in budgets], ctypes.c_int64),
                                _ptr_array([x.data_ptr() for x in idx]), n_sink, n_latent, span_width,
                                _stream_handle(stream))
+    if st != CB_OK:
+        raise CBError(st, lib.cb_last_error(None).decode())
+
+
+def select_noalloc_status(stream=None):
+    """cb_select_noalloc_status: wait for the stream and raise if the allocation-free selection's
+    kernel check failed since the last read."""
+    lib = load_library()
+    st = lib.cb_select_noalloc_status(_stream_handle(stream))
     if st != CB_OK:
         raise CBError(st, lib.cb_last_error(None).decode())
 
@@ -318,6 +331,11 @@ class CacheBack:
         self._check(self.lib.cb_gather(self.h, n, sp, Ta, src_stride, row_bytes, ip, Ca, out.data_ptr(),
                                        out.shape[0], Oa, out.stride(0) * out.element_size(),
                                        _stream_handle(stream)))
+
+    def set_wait_limit(self, limit_ns: int = 0, stall_next_score: bool = False):
+        """cb_set_wait_limit: limit of one bounded device wait (0: the 1 s default); with
+        stall_next_score the next tcgen05 cb_score makes one wait run out (failure-detection test)."""
+        self._check(self.lib.cb_set_wait_limit(self.h, int(limit_ns), 1 if stall_next_score else 0))
 
     STAGES = ("row_statistics", "statistics_combine", "normalised_accumulation", "finalize")
 

@@ -50,6 +50,8 @@ void stage_mark(StageTimer* t, int stage, cudaStream_t st) {
 }
 }  // namespace cbk
 
+constexpr int64_t kDefaultWaitNs = 1000000000;   // 1 s
+
 struct cb_ctx {
     cb_config cfg;
     int device = 0;
@@ -72,6 +74,8 @@ struct cb_ctx {
     int64_t keys_per_sender = 0;
     int64_t scratch_bytes = 0;
     int32_t score_path = 0;         // kernels of the last cb_score: 2 tcgen05, 1 mma.sync, 0 none yet
+    int64_t wait_ns = kDefaultWaitNs;   // limit of one bounded device wait (tcgen05 passes)
+    int32_t stall_next = 0;         // failure-detection test: stall the next cb_score once
     cbk::StageTimer* timer = nullptr;
     std::string last_error;
 };
@@ -430,6 +434,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->fin_cnt = ctx->fin_cnt;
         bt->stage = ctx->stage;
         bt->stage_elems = ctx->stage_elems;
+        bt->wait_ns = (uint64_t)ctx->wait_ns;
+        bt->stall = b0 == 0 ? ctx->stall_next : 0;
         int64_t so = 0, oo = 0, eo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
@@ -462,7 +468,20 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         delete bt;
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "score launch failed: %s", cudaGetErrorString(e));
     }
+    ctx->stall_next = 0;
     if (ctx->timer) ++ctx->timer->calls;
+    return CB_OK;
+}
+
+cb_status cb_set_wait_limit(cb_ctx* ctx, int64_t limit_ns, int32_t stall_next_score) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    if (limit_ns != 0 && (limit_ns < 1000 || limit_ns > 60000000000ll))
+        return fail(ctx, CB_EINVAL, "limit_ns = %lld: 0 (the default, 1 s) or 1e3 .. 6e10", (long long)limit_ns);
+    if (stall_next_score != 0 && stall_next_score != 1)
+        return fail(ctx, CB_EINVAL, "stall_next_score must be 0 or 1");
+    ctx->wait_ns = limit_ns ? limit_ns : kDefaultWaitNs;
+    ctx->stall_next = stall_next_score;
     return CB_OK;
 }
 

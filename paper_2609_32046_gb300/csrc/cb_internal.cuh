@@ -98,6 +98,8 @@ struct ScoreBatch {
     uint32_t* fin_cnt;        // finalize: finished slice blocks per tile (zero between launches)
     uint16_t* stage;          // tcgen05 passes: contiguous copies of paged senders' K
     int64_t stage_elems;      // its capacity (bf16 elements)
+    uint64_t wait_ns;         // tcgen05 passes: limit of one bounded mbarrier wait
+    int32_t stall;            // tcgen05 passes: failure-detection test (one wait nothing completes)
     ScoreSender s[kMaxBatch];
 };
 

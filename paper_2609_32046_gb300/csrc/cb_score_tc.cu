@@ -78,6 +78,8 @@ struct TcBatch {
     float sl2e, p;
     int32_t p_is_2, p_inf, ph;
     int64_t units1, units2;
+    uint64_t wait_ns;     // limit of one bounded mbarrier wait
+    int32_t stall;        // 1: CTA 0's pass-1 MMA issuer first waits on a barrier nothing arrives on
     uint32_t* err;
     TcSender s[kMaxTcSenders];
 };
@@ -87,6 +89,8 @@ struct Ctl {
     uint64_t t_full[4], t_empty[4];   // TMEM buffers of 128 columns (pass 1: group g owns 2g and 2g + 1;
                                       // pass 2: buffer 2g + h is column half h of group g)
     uint64_t q_full, q_empty, drain, o_full;
+    uint64_t stall;         // failure-detection test: a barrier nothing arrives on
+    uint64_t wait_ns;       // limit of one bounded wait
     uint64_t xb[2][2][4];   // pass 2: column-half exchange [tile parity][group][lane quarter]: written
     uint64_t xe[2][2][4];   //   and read (half 1 reuses a slot only after half 0 has read it)
     uint32_t tmem_base;
@@ -109,7 +113,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Ctl* ct
         if (mbar_try_wait_hint(bar, parity, kPollNs)) return true;
         if ((i & 63) == 0) {
             if (*reinterpret_cast<volatile int*>(&ctl->abort)) return false;
-            if (now_ns() - t0 > kWaitNs) {
+            if (now_ns() - t0 > ctl->wait_ns) {
                 *reinterpret_cast<volatile int*>(&ctl->abort) = 1;
                 atomicOr(err, kErrTimeout | (1u << (8 + tag)));
                 return false;
@@ -121,7 +125,8 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Ctl* ct
     return false;
 }
 
-// Wait used only on the way out (drain): bounded, ignores the abort flag.
+// Wait used only on the way out (drain): bounded by kWaitNs whatever the configured limit
+// (the copies and MMAs it waits for always complete), ignores the abort flag.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
     const uint64_t t0 = now_ns();
     while (!mbar_try_wait(bar, parity))
@@ -206,7 +211,7 @@ __device__ __forceinline__ Smem carve(uint8_t* raw, const TcBatch& bt) {
 
 // `releasers`: warps that arrive on a TMEM buffer's empty barrier (pass 1: the eight warps of a
 // group; pass 2: the four warps of one column half).
-__device__ __forceinline__ void init_ctl(Ctl* ctl, int stages, int releasers) {
+__device__ __forceinline__ void init_ctl(Ctl* ctl, int stages, int releasers, uint64_t wait_ns) {
     for (int k = 0; k < stages; ++k) {
         mbar_init(&ctl->k_full[k], 1);
         mbar_init(&ctl->k_empty[k], 1);
@@ -219,6 +224,8 @@ __device__ __forceinline__ void init_ctl(Ctl* ctl, int stages, int releasers) {
     mbar_init(&ctl->q_empty, 1);
     mbar_init(&ctl->drain, 1);
     mbar_init(&ctl->o_full, 1);
+    mbar_init(&ctl->stall, 1);
+    ctl->wait_ns = wait_ns;
     for (int k = 0; k < 16; ++k) {
         mbar_init(&ctl->xb[k >> 3][(k >> 2) & 1][k & 3], 1);
         mbar_init(&ctl->xe[k >> 3][(k >> 2) & 1][k & 3], 1);
@@ -302,7 +309,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
     const Smem sm = carve(smem_raw, bt);
     Ctl* ctl = sm.ctl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 8);
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 8, bt.wait_ns);
     if (warp == 1) {
         tmem_alloc(&ctl->tmem_base, kTmemCols);
         tmem_relinquish();
@@ -356,6 +363,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_stats_tc(const __grid_constan
             uint32_t ph = 0;
             int prev = -1;
             bool ok = true;
+            // failure-detection test: wait on a barrier that nothing arrives on, so the bounded
+            // wait gives up, sets the abort flag and every role of this CTA leaves
+            if (bt.stall && blockIdx.x == 0) ok = wait_bar(&ctl->stall, 0, ctl, bt.err, 6);
             Unit un = decode1(bt, ub);
             for (int64_t u = ub; u < ue && ok; ++u, next1(bt, un)) {
                 const TcSender& sd = bt.s[un.i];
@@ -567,7 +577,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
     const Smem sm = carve(smem_raw, bt);
     Ctl* ctl = sm.ctl;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 4);
+    if (threadIdx.x == 0) init_ctl(ctl, bt.stages, 4, bt.wait_ns);
     if (warp == 1) {
         tmem_alloc(&ctl->tmem_base, kTmemCols);
         tmem_relinquish();
@@ -1043,6 +1053,8 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
         tb->stages = rpad_max > 256 ? 2 : 4;
         tb->units1 = u1;
         tb->units2 = u2;
+        tb->wait_ns = b.wait_ns;
+        tb->stall = batches.size() == 1 ? b.stall : 0;   // the first launch only
     }
     cudaError_t e = cudaSuccess;
     for (size_t k = 0; k < batches.size() && e == cudaSuccess; ++k) {

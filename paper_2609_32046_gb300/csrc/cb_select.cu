@@ -441,7 +441,7 @@ extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, co
     cb_status st = CB_OK;
     int dev = 0;
     float* scratch = nullptr;
-    int64_t spans = 0;
+    set_context_free_error("");
     if (n < 1 || n > 4096) {
         snprintf(msg, sizeof msg, "n = %d not in [1, 4096]", n);
         st = CB_ESHAPE;
@@ -456,6 +456,10 @@ extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, co
         snprintf(msg, sizeof msg, "no CUDA device");
         st = CB_ECUDA;
     }
+    // Only senders with more than kSmemSpans spans keep their span means in the array (the
+    // kernel holds fewer in shared memory); each launch of up to kMaxBatch senders places its
+    // own such senders from slot 0, so the largest launch decides what the call needs.
+    int64_t group_slots = 0, max_slots = 0;
     for (int i = 0; st == CB_OK && i < n; ++i) {
         if (T[i] < 1 || T[i] > INT32_MAX) {
             snprintf(msg, sizeof msg, "T[%d] = %lld not in [1, 2^31)", i, (long long)T[i]);
@@ -471,13 +475,17 @@ extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, co
             st = CB_EBUDGET;
             break;
         }
-        spans += (T[i] + span_width - 1) / span_width;
+        if (i % kMaxBatch == 0) group_slots = 0;
+        const int64_t nsp = (T[i] + span_width - 1) / span_width;
+        if (nsp > kSmemSpans) group_slots += nsp;
+        max_slots = group_slots > max_slots ? group_slots : max_slots;
         if ((st = noalloc_check_ptr(scores[i], dev, "scores", i, msg, sizeof msg))) break;
         if ((st = noalloc_check_ptr(idx[i], dev, "idx", i, msg, sizeof msg))) break;
     }
-    if (st == CB_OK && spans > kNoAllocMaxSpans) {
-        snprintf(msg, sizeof msg, "the call needs %lld span slots; this entry point holds at most %lld "
-                 "(use cb_select with a context for larger calls)", (long long)spans, (long long)kNoAllocMaxSpans);
+    if (st == CB_OK && max_slots > kNoAllocMaxSpans) {
+        snprintf(msg, sizeof msg, "one launch of the call needs %lld span slots for senders of more than %d "
+                 "spans; this entry point holds at most %lld (use cb_select with a context for larger calls)",
+                 (long long)max_slots, kSmemSpans, (long long)kNoAllocMaxSpans);
         st = CB_ESHAPE;
     }
     if (st == CB_OK) st = noalloc_scratch(dev, &scratch, msg, sizeof msg);
@@ -500,12 +508,13 @@ extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, co
         bt.err = status_word;
         int64_t off = 0;
         for (int k = 0; k < nb; ++k) {
+            const int64_t nsp = (T[b0 + k] + span_width - 1) / span_width;
             bt.s[k].scores = scores[b0 + k];
             bt.s[k].idx = idx[b0 + k];
             bt.s[k].T = T[b0 + k];
             bt.s[k].B = budget[b0 + k];
-            bt.s[k].span_keys = scratch + off;
-            off += (T[b0 + k] + span_width - 1) / span_width;
+            bt.s[k].span_keys = nsp > kSmemSpans ? scratch + off : nullptr;   // else unused by the kernel
+            if (nsp > kSmemSpans) off += nsp;
         }
         e = launch_select(bt, strm);
     }
@@ -513,6 +522,45 @@ extern "C" cb_status cb_select_noalloc(int32_t n, const float* const* scores, co
         snprintf(msg, sizeof msg, "select launch failed: %s", cudaGetErrorString(e));
         set_context_free_error(msg);
         return CB_ECUDA;
+    }
+    return CB_OK;
+}
+
+extern "C" cb_status cb_select_noalloc_status(void* stream) {
+    using namespace cbk;
+    char msg[256] = "";
+    set_context_free_error("");
+    int dev = 0;
+    float* scratch = nullptr;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        set_context_free_error("no CUDA device");
+        return CB_ECUDA;
+    }
+    cb_status st = noalloc_scratch(dev, &scratch, msg, sizeof msg);
+    if (st != CB_OK) {
+        set_context_free_error(msg);
+        return st;
+    }
+    cudaStream_t strm = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t* status_word = reinterpret_cast<uint32_t*>(scratch + kNoAllocMaxSpans);
+    uint32_t word = 0;
+    cudaError_t e = cudaMemcpyAsync(&word, status_word, sizeof word, cudaMemcpyDeviceToHost, strm);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(strm);
+    if (e == cudaSuccess && word) {
+        e = cudaMemsetAsync(status_word, 0, sizeof(uint32_t), strm);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(strm);
+    }
+    if (e != cudaSuccess) {
+        snprintf(msg, sizeof msg, "device error: %s", cudaGetErrorString(e));
+        set_context_free_error(msg);
+        return CB_ECUDA;
+    }
+    if (word) {
+        snprintf(msg, sizeof msg, "the selection kernel's own check failed (code 0x%x:%s)", word,
+                 (word & kErrSelectBudget) ? " selected count differs from the budget" : "");
+        set_context_free_error(msg);
+        return CB_EDEVICE;
     }
     return CB_OK;
 }

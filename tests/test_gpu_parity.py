@@ -284,3 +284,72 @@ def test_extreme_logit_rows(kernel, scale):
     c.sync_status()
     assert c.score_path() == kernel
     check_sender(f, 0, K, V, Q)
+
+
+# Every pass-2 instantiation the tcgen05 path admits: k_accum_tc<G, pool_width / 2, p == 2>, G in
+# {1, 2, 4}, pool widths 1, 3, 5, 7 and p = 2 or not (p = 3 for the general power).
+TC_INSTANCES = [(G, pw, p) for G in (1, 2, 4) for pw in (1, 3, 5, 7) for p in (2.0, 3.0)]
+
+
+@pytest.mark.parametrize("G,pool_width,p", TC_INSTANCES,
+                         ids=["g%d_pool%d_p%g" % c for c in TC_INSTANCES])
+def test_tcgen05_every_instantiation(G, pool_width, p):
+    Hkv = 4
+    m = {1: 61, 2: 45, 4: 33}[G]            # 61, 90 and 132 query rows: one and two 128-row halves
+    w = synth.custom_workload(synth.Shape(2, G * Hkv, Hkv, 128), [431], m,
+                              seed=100 * G + 10 * pool_width + int(p), n_planted_spans=2)
+    extra = dict(pool_width=pool_width, p=p)
+    f = run_path(w, 0.3, score_kernel=2, **extra)
+    assert f.cb.score_path() == 2
+    s = w.senders[0]
+    check_sender(f, 0, s.K, s.V, w.queries[0], p=p, pool_w=pool_width)
+
+
+@pytest.mark.parametrize("G", [1, 2, 4])
+def test_tcgen05_unpooled_variance_identity(G):
+    """App. C.1: at p = 2 without pooling, C_t = 1 + sum_s Var_r(b) / sum_s (mean_r b)^2, and with
+    alpha = 1, S_t = Q_t C_t where Q_t = sum_s mean over (r, h) of a is the unpooled mean query
+    attention.  b comes from torch's fp64 softmax (not from the oracle), and the GPU scores of the
+    tcgen05 passes must satisfy the identity within the score tolerance."""
+    import math
+    nL, Hkv, T, m = 2, 4, 517, {1: 50, 2: 37, 4: 29}[G]
+    Hq = G * Hkv
+    w = synth.custom_workload(synth.Shape(nL, Hq, Hkv, 128), [T], m, seed=31 + G, n_planted_spans=3)
+    f = run_path(w, 0.25, score_kernel=2, pool_width=1, p=2.0, alpha=1.0)
+    assert f.cb.score_path() == 2
+    K, Q = w.senders[0].K, w.queries[0]
+    Qd = Q.to(torch.float64).permute(0, 2, 1, 3)                                  # [nL][Hq][m][d]
+    eye = torch.eye(T, dtype=torch.float64).expand(nL, Hkv, T, T)
+    a = torch.nn.functional.scaled_dot_product_attention(
+        Qd, K.to(torch.float64), eye, scale=1.0 / math.sqrt(128), enable_gqa=True).numpy()   # [nL][Hq][m][T]
+    b = a.reshape(nL, Hkv, G, m, T).mean(axis=2)                                  # [nL][Hkv][m][T]
+    C = 1.0 + b.var(axis=2).sum(axis=(0, 1)) / (b.mean(axis=2) ** 2).sum(axis=(0, 1))
+    U = a.sum(axis=(1, 2)).sum(axis=0) / (m * Hq)
+    assert_scores_close(f.scores[0].cpu().numpy(), U * C)
+
+
+def test_tcgen05_bounded_wait_gives_up_and_context_recovers():
+    """Failure detection without a GPU fault: one wait of the row-statistics kernel is made to
+    wait on a barrier nothing arrives on.  After the configured limit it gives up, the kernel
+    drains its copies and MMAs, frees its tensor memory and returns; the host reads CB_ETIMEOUT.
+    The same context then scores correctly."""
+    w = synth.custom_workload(synth.Shape(2, 32, 8, 128), [3000], 64, seed=41, n_planted_spans=2)
+    s = w.senders[0]
+    K, V, Q = s.K.cuda(), s.V.cuda(), w.queries[0].cuda()
+    c = make_cb(w.spec.shape, 3000, 64, 1, score_kernel=2)
+    S = torch.empty(3000, device="cuda")
+    c.set_wait_limit(20_000_000, stall_next_score=True)        # 20 ms
+    c.score([K], [Q], [S])
+    with pytest.raises(cb.CBError) as e:
+        c.sync_status()
+    assert e.value.status == cb.CB_ETIMEOUT
+    assert "gave up" in str(e.value)
+    c.sync_status()                                            # cleared
+    # the stall was for one call; the short limit stays and ordinary waits stay far below it
+    f = cb.Filter(c, [(K, V)], [Q], 0.25).run()
+    c.sync_status()
+    check_sender(f, 0, s.K, s.V, w.queries[0])
+    c.set_wait_limit(0)
+    with pytest.raises(cb.CBError) as e:
+        c.set_wait_limit(10)                                   # below 1 microsecond
+    assert e.value.status == cb.CB_EINVAL
