@@ -65,8 +65,6 @@ struct cb_ctx {
     uint16_t* ext = nullptr;        // tcgen05 passes: per-row offset terms [S][nS][R_pad][16] bf16
     uint16_t* ones = nullptr;       // tcgen05 passes: [128][16] bf16 block of ones columns
     float* part = nullptr;
-    float* fin = nullptr;
-    uint32_t* fin_cnt = nullptr;
     float* span_keys = nullptr;
     uint16_t* stage = nullptr;      // tcgen05 passes: contiguous copies of paged senders' K (on demand)
     int64_t stage_elems = 0;
@@ -297,13 +295,6 @@ cb_status cb_create(const cb_config* cfg, cb_ctx** out) {
     e = alloc(&ctx->stats, (size_t)(S * nS * ctx->n_chunk1_max * rows), &total);
     if (e == cudaSuccess) e = alloc(&ctx->offs, (size_t)(S * nS * rows), &total);
     if (e == cudaSuccess) e = alloc(&ctx->part, (size_t)(S * 3 * nS * c.max_positions), &total);
-    if (e == cudaSuccess) e = alloc(&ctx->fin, (size_t)(S * cbk::finalize_floats(c.max_positions)), &total);
-    if (e == cudaSuccess) {
-        // one launch holds at most kMaxBatch senders; counters return to zero after each launch
-        const int64_t nb = S < cbk::kMaxBatch ? S : cbk::kMaxBatch;
-        e = alloc(&ctx->fin_cnt, (size_t)(nb * cbk::finalize_tiles(c.max_positions)), &total);
-        if (e == cudaSuccess) e = cudaMemset(ctx->fin_cnt, 0, (size_t)(nb * cbk::finalize_tiles(c.max_positions)) * 4);
-    }
     if (e == cudaSuccess) e = alloc(&ctx->span_keys, (size_t)(S * ctx->keys_per_sender), &total);
     if (e == cudaSuccess && ctx->use_tc) {
         e = alloc(&ctx->ext, (size_t)(S * nS * cbk::rows_pad128(rows) * cbk::kExtCols), &total);
@@ -338,8 +329,6 @@ void cb_destroy(cb_ctx* ctx) {
         cudaFree(ctx->ext);
         cudaFree(ctx->ones);
         cudaFree(ctx->part);
-        cudaFree(ctx->fin);
-        cudaFree(ctx->fin_cnt);
         cudaFree(ctx->span_keys);
         cudaFree(ctx->stage);
         cudaFree(ctx->err);
@@ -430,13 +419,11 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
         bt->ext = ctx->use_tc ? ctx->ext : nullptr;
         bt->ones = ctx->ones;
         bt->part = ctx->part;
-        bt->fin = ctx->fin;
-        bt->fin_cnt = ctx->fin_cnt;
         bt->stage = ctx->stage;
         bt->stage_elems = ctx->stage_elems;
         bt->wait_ns = (uint64_t)ctx->wait_ns;
         bt->stall = b0 == 0 ? ctx->stall_next : 0;
-        int64_t so = 0, oo = 0, eo = 0, po = 0, fo = 0, b1 = 0, b2 = 0;
+        int64_t so = 0, oo = 0, eo = 0, po = 0, b1 = 0, b2 = 0;
         for (int k = 0; k < nb; ++k) {
             const cb_kv& s = senders[b0 + k];
             const cb_query& q = queries[b0 + k];
@@ -457,10 +444,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.offs_off = oo; oo += (int64_t)nS * q.m * ctx->G;
             d.ext_off = eo; eo += (int64_t)nS * cbk::rows_pad128((int64_t)q.m * ctx->G) * cbk::kExtCols;
             d.part_off = po; po += (int64_t)3 * nS * s.T;
-            d.fin_off = fo; fo += cbk::finalize_floats(s.T);
             d.blk1_begin = b1; b1 += (int64_t)nS * d.n_chunk1;
             d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
-            d.blkf_begin = 0;  // set by the score launcher
         }
         int path = 0;
         cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms, &path);

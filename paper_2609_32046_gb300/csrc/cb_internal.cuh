@@ -72,10 +72,8 @@ struct ScoreSender {
     int64_t offs_off;         // float offset of this sender's per-row softmax offsets
     int64_t ext_off;          // bf16 offset of this sender's [nS][R_pad][16] offset rows (tcgen05 passes)
     int64_t part_off;         // float offset of this sender's [3][nS][T] partials
-    int64_t fin_off;          // float offset of this sender's finalize slice sums (finalize_floats(T))
     int64_t blk1_begin;       // first pass-1 block of this sender
     int64_t blk2_begin;       // first pass-2 block of this sender
-    int64_t blkf_begin;       // first finalize tile of this sender (its counters start there)
 };
 
 struct ScoreBatch {
@@ -94,8 +92,6 @@ struct ScoreBatch {
                               // (hi, mid, lo, then 13 zeros; -1e30 on padding rows), else null
     const uint16_t* ones;     // tcgen05 passes: [128][16] bf16, columns 0-2 = 1, the rest 0
     float* part;              // per-group U_s, N_s, D_s partials
-    float* fin;               // finalize slice sums [sender][tile][kFinSlices][3][256]
-    uint32_t* fin_cnt;        // finalize: finished slice blocks per tile (zero between launches)
     uint16_t* stage;          // tcgen05 passes: contiguous copies of paged senders' K
     int64_t stage_elems;      // its capacity (bf16 elements)
     uint64_t wait_ns;         // tcgen05 passes: limit of one bounded mbarrier wait
@@ -187,8 +183,6 @@ struct GatherBatch {
 void set_context_free_error(const char* msg);
 
 // Finalize tiles of a sender of T positions, and the floats of its slice sums.
-int64_t finalize_tiles(int64_t T);
-int64_t finalize_floats(int64_t T);
 
 // True when the tcgen05 score passes handle this shape.
 bool tc_path_supported(int head_dim, int G, int pool_half, int max_query_tokens);

@@ -517,103 +517,133 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // finalize: fixed-order sums over the groups, Pool(U), C, S -- one launch
 // ---------------------------------------------------------------------------
-// Block (tile, slice k, sender) covers the tile's 256 positions: 240 outputs and kHalo on each
-// side for Pool.  It sums slice k of the groups (s = k, k + 16, ...) in increasing order per
-// position (U everywhere, N and D at the outputs) into the tile's slice buffer, then counts
-// itself done on the tile's counter.  The last of the tile's 16 slice blocks adds the 16 slice
-// sums in slice order, pools U and writes C and S, and resets the counter for the next call.
-// The order of every sum is fixed, so the result does not depend on which block is last.
-constexpr int kFinBlock = 256;
-constexpr int kFinOut2 = kFinBlock - 2 * kHalo;        // outputs per tile
+// Block (64-position tile, sender); thread (slice k, quad q) sums slice k of the groups
+// (s = k, k + 16, ... in increasing order) for the four consecutive positions of quad q:
+// quads 2..17 are the tile (U, N and D), quads 0, 1 and 18, 19 the kHalo positions on each
+// side (U only, for Pool).  Nine groups' loads are issued before they are added (the partials
+// mostly come from DRAM, so the kernel needs many bytes in flight), with one 16-byte load per
+// quad where the sender's partial rows are 16-byte aligned.  The 16 slice sums of every
+// position are then added in slice order in shared memory, U is pooled and C and S written.
+// Each sum has a fixed order, so the scores are deterministic.
+constexpr int kFinPos = 64;                          // output positions per block
+constexpr int kFinQuads = kFinPos / 4 + kHalo / 2;   // 16 tile quads + 2 on each side
+constexpr int kFinSpan = 4 * kFinQuads;              // positions whose U is summed
+constexpr int kFinThreads = kFinSlices * kFinQuads;  // 320
+constexpr int kFinBatch = 9;                         // groups loaded before they are added
 
-__global__ void __launch_bounds__(kFinBlock) k_finalize(const __grid_constant__ ScoreBatch bt) {
-    __shared__ float us[kFinBlock];
-    __shared__ int last;
-    const ScoreSender& sd = bt.s[blockIdx.z];
+__global__ void __launch_bounds__(kFinThreads) k_finalize(const __grid_constant__ ScoreBatch bt) {
+    __shared__ float su[kFinSlices][kFinSpan];
+    __shared__ float sn[kFinSlices][kFinPos];
+    __shared__ float sdn[kFinSlices][kFinPos];
+    __shared__ float us[kFinSpan];
+    const ScoreSender& sd = bt.s[blockIdx.y];
     const int64_t T = sd.T;
-    const int64_t tile = blockIdx.x;
-    if (tile * kFinOut2 >= T) return;
-    const int sl = blockIdx.y;
+    const int64_t t0 = (int64_t)blockIdx.x * kFinPos;
+    if (t0 >= T) return;
+    const int sl = threadIdx.x / kFinQuads, q = threadIdx.x % kFinQuads;
     const int nS = bt.n_layers * bt.n_kv_heads;
-    const int lp = threadIdx.x;
-    const int64_t t = tile * kFinOut2 - kHalo + lp;
-    const bool inside = (t >= 0 && t < T);
-    const bool centre = lp >= kHalo && lp < kFinBlock - kHalo;
-    float* fin = bt.fin + sd.fin_off + tile * (kFinSlices * 3 * kFinBlock);   // [slice][3][256]
-    {
-        float U = 0.f, Nv = 0.f, Dv = 0.f;   // p = infinity: N and D are maxima over the groups (all >= 0)
-        if (inside) {
-            const float* part = bt.part + sd.part_off + t;
-            if (!centre) {
-#pragma unroll 18
-                for (int s = sl; s < nS; s += kFinSlices) U += __ldcs(part + (int64_t)s * T);
-            } else if (bt.p_inf) {
-#pragma unroll 18
-                for (int s = sl; s < nS; s += kFinSlices) {
-                    U += __ldcs(part + (int64_t)s * T);
-                    Nv = fmaxf(Nv, __ldcs(part + ((int64_t)nS + s) * T));
-                    Dv = fmaxf(Dv, __ldcs(part + ((int64_t)2 * nS + s) * T));
+    const float* part = bt.part + sd.part_off;
+    const int64_t rN = (int64_t)nS * T, rD = 2 * rN;    // first N and D rows
+    const bool pinf = bt.p_inf;
+    const bool full = q >= kHalo / 4 && q < kHalo / 4 + kFinPos / 4;   // a tile quad: N and D too
+    const int64_t t = t0 - kHalo + 4 * q;
+    float u[4] = {0.f, 0.f, 0.f, 0.f}, n[4] = {0.f, 0.f, 0.f, 0.f}, d[4] = {0.f, 0.f, 0.f, 0.f};
+    auto add = [&](float (&acc)[4], const float4 v, bool mx) {
+        if (mx) {
+            acc[0] = fmaxf(acc[0], v.x); acc[1] = fmaxf(acc[1], v.y);
+            acc[2] = fmaxf(acc[2], v.z); acc[3] = fmaxf(acc[3], v.w);
+        } else {
+            acc[0] += v.x; acc[1] += v.y; acc[2] += v.z; acc[3] += v.w;
+        }
+    };
+    if ((T & 3) == 0 && (sd.part_off & 3) == 0) {
+        // 16-byte aligned rows: the quad lies wholly inside or wholly outside [0, T)
+        if (t >= 0 && t < T) {
+            const float4* p = reinterpret_cast<const float4*>(part + t);
+            const int64_t rs = T / 4;   // row stride in float4
+            for (int s0 = sl; s0 < nS; s0 += kFinSlices * kFinBatch) {
+                float4 a[kFinBatch], b[kFinBatch], c[kFinBatch];
+#pragma unroll
+                for (int k = 0; k < kFinBatch; ++k) {
+                    const int s = s0 + k * kFinSlices;
+                    if (s < nS) {
+                        a[k] = __ldcs(p + (int64_t)s * rs);
+                        if (full) {
+                            b[k] = __ldcs(p + (rN / 4) + (int64_t)s * rs);
+                            c[k] = __ldcs(p + (rD / 4) + (int64_t)s * rs);
+                        }
+                    }
                 }
-            } else {
-#pragma unroll 18
-                for (int s = sl; s < nS; s += kFinSlices) {
-                    U += __ldcs(part + (int64_t)s * T);
-                    Nv += __ldcs(part + ((int64_t)nS + s) * T);
-                    Dv += __ldcs(part + ((int64_t)2 * nS + s) * T);
+#pragma unroll
+                for (int k = 0; k < kFinBatch; ++k) {
+                    if (s0 + k * kFinSlices >= nS) break;
+                    add(u, a[k], false);
+                    if (full) {
+                        add(n, b[k], pinf);   // p = infinity: N and D are maxima over the groups
+                        add(d, c[k], pinf);
+                    }
                 }
             }
         }
-        float* f = fin + sl * 3 * kFinBlock + lp;
-        f[0] = U;
-        f[kFinBlock] = Nv;
-        f[2 * kFinBlock] = Dv;
-    }
-    __threadfence();
-    __syncthreads();
-    uint32_t* cnt = bt.fin_cnt + sd.blkf_begin + tile;
-    if (lp == 0) last = atomicAdd(cnt, 1u) == kFinSlices - 1;
-    __syncthreads();
-    if (!last) return;
-    __threadfence();
-    float U = 0.f, Nv = 0.f, Dv = 0.f;
-    if (inside) {
+    } else {
 #pragma unroll
-        for (int k = 0; k < kFinSlices; ++k) U += __ldcg(fin + k * 3 * kFinBlock + lp);
-        if (centre) {
-#pragma unroll
-            for (int k = 0; k < kFinSlices; ++k) {
-                const float n_k = __ldcg(fin + (k * 3 + 1) * kFinBlock + lp);
-                const float d_k = __ldcg(fin + (k * 3 + 2) * kFinBlock + lp);
-                Nv = bt.p_inf ? fmaxf(Nv, n_k) : Nv + n_k;
-                Dv = bt.p_inf ? fmaxf(Dv, d_k) : Dv + d_k;
+        for (int e = 0; e < 4; ++e) {
+            const int64_t te = t + e;
+            if (te < 0 || te >= T) continue;   // outside the sender: U = 0 adds nothing to Pool
+            const float* p = part + te;
+            for (int s = sl; s < nS; s += kFinSlices) {
+                u[e] += __ldcs(p + (int64_t)s * T);
+                if (!full) continue;
+                const float b = __ldcs(p + rN + (int64_t)s * T), c = __ldcs(p + rD + (int64_t)s * T);
+                n[e] = pinf ? fmaxf(n[e], b) : n[e] + b;
+                d[e] = pinf ? fmaxf(d[e], c) : d[e] + c;
             }
         }
     }
-    us[lp] = U;
-    if (lp == 0) *cnt = 0u;   // every slice block of this tile has counted itself
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        su[sl][4 * q + e] = u[e];
+        if (full) {
+            sn[sl][4 * q - kHalo + e] = n[e];
+            sdn[sl][4 * q - kHalo + e] = d[e];
+        }
+    }
     __syncthreads();
-    if (centre && inside) {
+    const int x = threadIdx.x;
+    if (x < kFinSpan) {
+        float U = 0.f;
+#pragma unroll
+        for (int k = 0; k < kFinSlices; ++k) U += su[k][x];
+        us[x] = U;
+    }
+    float Nv = 0.f, Dv = 0.f;
+    if (x < kFinPos) {
+#pragma unroll
+        for (int k = 0; k < kFinSlices; ++k) {
+            Nv = pinf ? fmaxf(Nv, sn[k][x]) : Nv + sn[k][x];
+            Dv = pinf ? fmaxf(Dv, sdn[k][x]) : Dv + sdn[k][x];
+        }
+    }
+    __syncthreads();
+    if (x < kFinPos && t0 + x < T) {
         const int ph = bt.pool_half;
-        float Q = us[lp - ph];
-        for (int u = -ph + 1; u <= ph; ++u) Q = fmaxf(Q, us[lp + u]);
-        const float C = Dv > FLT_MIN ? (bt.p_inf ? Nv / Dv : powf(Nv / Dv, 1.f / (bt.p - 1.f))) : 1.f;
-        const float S = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
-        sd.scores[t] = S;
+        const int c = x + kHalo;
+        float Q = us[c - ph];
+        for (int v = -ph + 1; v <= ph; ++v) Q = fmaxf(Q, us[c + v]);
+        const float C = Dv > FLT_MIN ? (pinf ? Nv / Dv : powf(Nv / Dv, 1.f / (bt.p - 1.f))) : 1.f;
+        sd.scores[t0 + x] = bt.alpha == 0.f ? Q : Q * powf(C, bt.alpha);
     }
 }
 
 }  // namespace
-
-int64_t finalize_tiles(int64_t T) { return (T + kFinOut2 - 1) / kFinOut2; }
-int64_t finalize_floats(int64_t T) { return finalize_tiles(T) * kFinSlices * 3 * kFinBlock; }
 
 namespace {
 
 cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
     int64_t maxT = 0;
     for (int i = 0; i < b.n; ++i) maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
-    dim3 grid((unsigned)finalize_tiles(maxT), kFinSlices, (unsigned)b.n);
-    k_finalize<<<grid, kFinBlock, 0, st>>>(b);
+    dim3 grid((unsigned)((maxT + kFinPos - 1) / kFinPos), (unsigned)b.n);
+    k_finalize<<<grid, kFinThreads, 0, st>>>(b);
     return cudaGetLastError();
 }
 
@@ -644,13 +674,12 @@ size_t accum_smem(int max_rows) {
 
 template <int D, int G>
 cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
-    int64_t nblk1 = 0, nblk2 = 0, nblkf = 0;
+    int64_t nblk1 = 0, nblk2 = 0;
     int max_rows = 0;
     const int nS = b.n_layers * b.n_kv_heads;
     for (int i = 0; i < b.n; ++i) {
         nblk1 += (int64_t)nS * b.s[i].n_chunk1;
         nblk2 += (int64_t)nS * b.s[i].n_chunk2;
-        nblkf += finalize_tiles(b.s[i].T);
         max_rows = max_rows > b.s[i].m * G ? max_rows : b.s[i].m * G;
     }
     const size_t smem1 = (size_t)kStatsChunk * D * 2;
@@ -678,15 +707,7 @@ cudaError_t launch_score_tc(ScoreBatch& b, cudaStream_t st, int num_sms, uint32_
 
 cudaError_t launch_score(const ScoreBatch& b_in, cudaStream_t st, int num_sms, int* path_out) {
     const int G = b_in.n_q_heads / b_in.n_kv_heads;
-    // finalize block ranges follow this file's finalize tile
-    ScoreBatch* bp = new ScoreBatch(b_in);
-    int64_t bf = 0;
-    for (int i = 0; i < bp->n; ++i) {
-        bp->s[i].blkf_begin = bf;
-        bf += finalize_tiles(bp->s[i].T);
-    }
-    const ScoreBatch& b = *bp;
-    struct Free { ScoreBatch* p; ~Free() { delete p; } } guard{bp};
+    const ScoreBatch& b = b_in;
     if (b.use_tc) {
         ScoreBatch* w = new ScoreBatch(b);
         cudaError_t e = launch_score_tc(*w, st, num_sms, b.err, launch_combine);
