@@ -248,17 +248,18 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // combine: per-row log2 offset = max + log2(sum) + log2(G) over all chunks
 // ---------------------------------------------------------------------------
-// Block = 64 rows x 4 slot lanes of one (sender, group s): slot lane j merges partial slots
-// j, j + 4, ... of its row with an online max/sum, then slot lane 0 merges the four results
-// in lane order (a fixed order, so the offsets are deterministic).
-constexpr int kCombRows = 64;
-__global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
-    __shared__ float2 part[4][kCombRows];
+// Thread = row of one (sender, group s).  Its partial slots are merged as four chains
+// (slots j, j + 4, j + 8, ... for j = 0..3, each with an online max / sum in slot order), then
+// the four chain results in chain order: a fixed order, so the offsets are deterministic.  All
+// slots of a batch of 32 are loaded before any is merged (the partials mostly come from DRAM),
+// and one thread a row keeps the whole grid in one wave.
+constexpr int kCombRows = 256;     // rows (threads) per block
+constexpr int kCombBatch = 32;     // slots loaded before they are merged
+__global__ void __launch_bounds__(kCombRows) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
     const int nS = bt.n_layers * bt.n_kv_heads;
-    const ScoreSender* sdp = nullptr;
     int i = 0;
     int64_t blk = blockIdx.x;
-    // blocks are laid out sender by sender, nS * ceil(R_pad / 64) of them per sender
+    // blocks are laid out sender by sender, nS * ceil(rows / 256) of them per sender
     for (; i < bt.n; ++i) {
         const int R_i = bt.s[i].m * G;
         const int rows_i = bt.ext ? (int)rows_pad128(R_i) : R_i;
@@ -267,15 +268,13 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
         blk -= nb;
     }
     if (i >= bt.n) return;
-    sdp = &bt.s[i];
-    const ScoreSender& sd = *sdp;
+    const ScoreSender& sd = bt.s[i];
     const int R = sd.m * G;
     const int rows = bt.ext ? (int)rows_pad128(R) : R;
     const int nrb = (rows + kCombRows - 1) / kCombRows;
     const int s = (int)(blk / nrb);
-    const int row = (int)(blk % nrb) * kCombRows + (threadIdx.x & (kCombRows - 1));
-    const int j = threadIdx.x / kCombRows;   // slot lane 0..3
-    const int lr = threadIdx.x & (kCombRows - 1);
+    const int row = (int)(blk % nrb) * kCombRows + threadIdx.x;
+    if (row >= rows) return;
     const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
     const int r_tok = row / G, hh = row - r_tok * G;
     const uint16_t* qrow = sd.q + (int64_t)l * sd.qs_l + (int64_t)r_tok * sd.qs_t + (int64_t)(g * G + hh) * sd.qs_h;
@@ -303,70 +302,63 @@ __global__ void __launch_bounds__(kThreads) k_combine(const __grid_constant__ Sc
         }
         return dot;
     };
-    // the query tokens' own keys: row (token r, head h) also attends to query keys 0..r (every
-    // fourth one on this slot lane); logits in the statistics' log2 domain
-    auto merge_self_keys = [&](float& M, float& L) {
-        for (int u = j; u <= r_tok; u += 4)
-            merge_logit(dot_row(sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h) *
-                            bt.scale_log2e, M, L);
+    // the query tokens' own keys: row (token r, head h) also attends to query keys 0..r, key u
+    // on chain u mod 4 (each chain in increasing u); logits in the statistics' log2 domain
+    auto merge_self_keys = [&](float (&M)[4], float (&L)[4]) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            for (int u = j; u <= r_tok; u += 4)
+                merge_logit(dot_row(sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h) *
+                                bt.scale_log2e, M[j], L[j]);
     };
-    float M = -INFINITY, L = 0.f;
+    float off = 0.f;
     if (row < R) {
+        float M[4], L[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) { M[j] = -INFINITY; L[j] = 0.f; }
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
-        // slots j, j + 4, j + 8, ... merged in that order; eight loads issued before each merge run
-        for (int c0 = j; c0 < sd.n_chunk1; c0 += 32) {
-            float2 vv[8];
+        for (int c0 = 0; c0 < sd.n_chunk1; c0 += kCombBatch) {
+            float2 vv[kCombBatch];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int c = c0 + 4 * q;
-                vv[q] = c < sd.n_chunk1 ? st[(int64_t)c * R] : make_float2(-INFINITY, 0.f);
-            }
+            for (int q = 0; q < kCombBatch; ++q)
+                vv[q] = c0 + q < sd.n_chunk1 ? st[(int64_t)(c0 + q) * R] : make_float2(-INFINITY, 0.f);
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
+            for (int q = 0; q < kCombBatch; ++q) {
                 const float2 v = vv[q];
+                const int j = q & 3;   // slot c0 + q is on chain (c0 + q) mod 4, c0 a multiple of 32
                 if (v.x == -INFINITY) continue;
-                if (v.x > M) {
-                    L = (M == -INFINITY ? 0.f : L * ex2(M - v.x)) + v.y;
-                    M = v.x;
+                if (v.x > M[j]) {
+                    L[j] = (M[j] == -INFINITY ? 0.f : L[j] * ex2(M[j] - v.x)) + v.y;
+                    M[j] = v.x;
                 } else {
-                    L += v.y * ex2(v.x - M);
+                    L[j] += v.y * ex2(v.x - M[j]);
                 }
             }
         }
         if (sd.kself) merge_self_keys(M, L);
-    }
-    // A chunk partial whose sum left fp32 range makes the row's sum infinite (pass 1 of the
-    // tensor-memory path offsets each chunk by the maximum of its first 32 logits, so a logit far
-    // larger later in the chunk overflows exp2).  Such rows, rare, are recomputed here from Q and
-    // K directly: the four slot lanes take every fourth sender position.
-    __shared__ int bad[4][kCombRows];
-    part[j][lr] = make_float2(M, L);
-    bad[j][lr] = row < R && !(L <= FLT_MAX);
-    __syncthreads();
-    if (row < R && (bad[0][lr] | bad[1][lr] | bad[2][lr] | bad[3][lr])) {
-        M = -INFINITY;
-        L = 0.f;
-        const uint16_t* kbase = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
-        for (int64_t t = j; t < sd.T; t += 4) {
-            const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
-            merge_logit(ro < 0 ? 0.f : dot_row(kbase + ro) * bt.scale_log2e, M, L);   // a bad page reads as zeros
+        // A chunk partial whose sum left fp32 range makes the row's sum infinite (pass 1 of the
+        // tensor-memory path offsets each chunk by the maximum of its first 32 logits, so a logit
+        // far larger later in the chunk overflows exp2).  Such rows, rare, are recomputed here
+        // from Q and K directly: position t on chain t mod 4.
+        if (!(L[0] <= FLT_MAX) || !(L[1] <= FLT_MAX) || !(L[2] <= FLT_MAX) || !(L[3] <= FLT_MAX)) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) { M[j] = -INFINITY; L[j] = 0.f; }
+            const uint16_t* kbase = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                for (int64_t t = j; t < sd.T; t += 4) {
+                    const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
+                    merge_logit(ro < 0 ? 0.f : dot_row(kbase + ro) * bt.scale_log2e, M[j], L[j]);   // a bad page reads as zeros
+                }
+            if (sd.kself) merge_self_keys(M, L);
         }
-        if (sd.kself) merge_self_keys(M, L);
-        part[j][lr] = make_float2(M, L);
-    }
-    __syncthreads();
-    if (j != 0 || row >= rows) return;
-    float off = 0.f;
-    if (row < R) {
         float Mx = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) Mx = fmaxf(Mx, part[k][threadIdx.x].x);
+        for (int k = 0; k < 4; ++k) Mx = fmaxf(Mx, M[k]);
         float Lx = 0.f;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float2 v = part[k][threadIdx.x];
-            if (v.x != -INFINITY) Lx += v.y * ex2(v.x - Mx);
-        }
+        for (int k = 0; k < 4; ++k)
+            if (M[k] != -INFINITY) Lx += L[k] * ex2(M[k] - Mx);
         off = Mx + log2f(Lx) + log2f((float)G);
         bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
     }
@@ -661,7 +653,7 @@ int64_t combine_blocks(const ScoreBatch& b) {
 
 cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
     const int G = b.n_q_heads / b.n_kv_heads;
-    k_combine<<<(unsigned)combine_blocks(b), kThreads, 0, st>>>(b, G);
+    k_combine<<<(unsigned)combine_blocks(b), kCombRows, 0, st>>>(b, G);
     return cudaGetLastError();
 }
 
@@ -691,7 +683,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     stage_mark(b.timer, kStageStart, st);
     k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
     stage_mark(b.timer, kStageStats, st);
-    k_combine<<<(unsigned)combine_blocks(b), kThreads, 0, st>>>(b, G);
+    k_combine<<<(unsigned)combine_blocks(b), kCombRows, 0, st>>>(b, G);
     stage_mark(b.timer, kStageCombine, st);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
     stage_mark(b.timer, kStageAccum, st);

@@ -814,13 +814,14 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_accum_tc(const __grid_constan
             const bool p_inf = !P2 && bt.p_inf;
             float nacc = p_inf ? fmaxf(nacc2[0], nacc2[1]) : nacc2[0] + nacc2[1];
             float bsum = bsum2[0] + bsum2[1];
-            // the two column halves of the group add up their sums; half 0 writes the results
+            // the two column halves of the group add up their sums; half tp (the group's tile
+            // parity) writes the results, so the halves take turns waiting for each other
             const int tp = (int)(gt & 1);
             float2* xs = xch + ((tp * 2 + grp) * 4 + sp) * 32;
             uint64_t* xb = &ctl->xb[tp][grp][sp];
             uint64_t* xe = &ctl->xe[tp][grp][sp];
-            if (hf == 1) {
-                // the slot was last used two tiles ago: wait until half 0 has read it
+            if ((hf ^ tp) == 1) {
+                // the slot was last used two tiles ago: wait until the other half has read it
                 if (!(ok = wait_bar(xe, (uint32_t)(((gt >> 1) & 1) ^ 1), ctl, bt.err, 7))) break;
                 xs[lane] = make_float2(nacc, bsum);
                 __syncwarp();
