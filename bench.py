@@ -68,6 +68,21 @@ def workload_bytes_flops(spec, keep):
     return tot_b, score_b, compact_b, tot_f
 
 
+def workload_config(spec, keep, paged: int = 0, ws: int = 1):
+    """The keys that define the workload of a bench line; both arms report the same dict."""
+    sh = spec.shape
+    states = 1 if spec.shared_sender else spec.n_senders
+    kv = sum(2 * sh.n_layers * sh.n_kv_heads * spec.T[i % len(spec.T)] * sh.head_dim * 2 for i in range(states))
+    l2 = ("inputs larger than L2 (K+V %.2f GB per rank), no flush" % (kv / 1e9)) if kv > 129e6 else \
+        "inputs within L2 (K+V %.1f MB): a parity size, not a timing configuration" % (kv / 1e6)
+    return {"workload": spec.name, "senders": spec.n_senders, "T": list(spec.T[:3]), "m": spec.m,
+            "n_layers": sh.n_layers, "q_heads": sh.n_q_heads, "kv_heads": sh.n_kv_heads,
+            "head_dim": sh.head_dim, "keep": keep,
+            "layout": ("paged: %d positions per page, pages in a random order" % paged) if paged
+            else "strided [nL][Hkv][T][d]",
+            "parallelism": "replicas" if ws > 1 else "single", "l2": l2}
+
+
 _REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
             0x80: "hw_power_brake_slowdown"}
 
@@ -272,7 +287,7 @@ def _oracle_inputs(spec_name: str, seed: int):
     return _ORACLE_INPUTS[key]
 
 
-def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
+def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0, keep=None):
     """Time the oracle on sender 0 of the workload, scoring n_layers_sample of its layers
     (0: sample_layers(spec)).
 
@@ -287,7 +302,7 @@ def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
     o = oracle.default()
     snd, Q = _oracle_inputs(spec_name, seed)
     nl = min(n_layers_sample, spec.shape.n_layers)
-    keep = spec.keeps[len(spec.keeps) // 2] if len(spec.keeps) > 1 else spec.keeps[0]
+    keep = spec.keeps[0] if keep is None else keep
     t0 = time.perf_counter()
     r = o.score(snd.K[:nl].contiguous(), Q[:nl].contiguous())
     t1 = time.perf_counter()
@@ -320,37 +335,44 @@ def oracle_sample(spec_name: str, n_layers_sample: int = 0, seed: int = 0):
 
 
 def run_reference(args):
+    """The reference arm: the fp64 C oracle on the host cores.  Each step scores a sample of the
+    workload (a ninth of the baseline's layers of sender 0: ~0.3 s on 16 cores for qwen8b) and
+    runs the full select and compact; `ms_per_step` is the measured wall time of that sample and
+    `value` the workload's tokens/s extrapolated from it (scoring is linear in the layers and
+    senders), with the factor in `extrapolation`."""
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     import oracle
     oracle.build()
-    vals = []
-    # each step a short sample (a ninth of the baseline's layers: ~0.3 s on 16 cores for
-    # qwen8b), so that --steps K --warmup W stays within a few minutes for the usual K
-    spec0 = synth_spec(args.workload)
-    layers = max(1, sample_layers(spec0) // 9) if not args.cpu_layers else args.cpu_layers
-    for k in range(args.warmup + args.steps):
-        r = oracle_sample(args.workload, layers)
-        if k >= args.warmup:
-            vals.append(r)
-    v = statistics.median([x["value"] for x in vals])
-    per_step_s = None
     import synth
     spec = synth.SPECS[args.workload]
+    layers = max(1, sample_layers(spec) // 9) if not args.cpu_layers else args.cpu_layers
+    layers = min(layers, spec.shape.n_layers)
+    keep = args.keep if args.keep is not None else spec.keeps[0]
+    vals, secs = [], []
+    for k in range(args.warmup + args.steps):
+        r = oracle_sample(args.workload, layers, keep=keep)
+        if k >= args.warmup:
+            vals.append(r)
+            secs.append(sum(r["seconds"].values()))   # the sample's score, select and compact
+    v = statistics.median([x["value"] for x in vals])
+    step_s = statistics.median(secs)
     tokens = sum(spec.T[i % len(spec.T)] for i in range(spec.n_senders))
-    per_step_s = tokens / v
     cpu = dict(vals[0])
     cpu["value"] = v
     cpu.pop("seconds", None)
     out = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": per_step_s * 1e3, "higher_is_better": True,
+           "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": args.workload, "senders": spec.n_senders, "T": list(spec.T[:3]), "m": spec.m,
-                      "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
-                      "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": spec.keeps[0],
-                      "layout": "strided [nL][Hkv][T][d]", "parallelism": "single"},
+           "config": workload_config(spec, keep),
+           "extrapolation": {"layers_scored": layers, "layers": spec.shape.n_layers, "senders_scored": 1,
+                             "senders": spec.n_senders, "tokens": tokens,
+                             "seconds_per_workload": tokens / v,
+                             "note": "each step scores sender 0 on layers_scored of its layers and runs the full "
+                                     "select and compact; value = the workload's tokens / (the measured score "
+                                     "time x layers / layers_scored x senders + select and compact x senders)"},
            "cpu_baseline": cpu,
            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
@@ -380,6 +402,91 @@ def paged_cache(cb, K, V, P: int, seed: int = 0):
             pool[:, order[b0:b1]] = blk.view(nL, Hkv, b1 - b0, P, d).permute(0, 2, 3, 1, 4)
         pools.append(pool)
     return cb.PagedKV(pools[0], pools[1], order.to(torch.int32), T)
+
+
+# the other Qwen3-8B-shaped workloads in the default line: (keep, timed steps, warm-up steps, peak)
+EXTRA_WORKLOADS = {"fanin": (0.25, 20, 3, "burst"), "hybrid": (0.10, 50, 3, "burst"),
+                   "sweep": (0.25, 6, 3, "sustained")}
+
+
+def time_workload(name: str, ws: int, rank: int, dev, use_graph: bool):
+    """One workload timed like the headline's steps (score + select + compact of every sender,
+    inputs resident, the timed steps replayed as one CUDA graph, clocks sampled in the timed
+    region, events around the second logit pass), then freed.  The sweep's steps run for ~0.1 s,
+    so its tensor roofline uses the sustained bf16 peak."""
+    import torch
+    import paper_2609_32046_gb300 as cb
+    import synth
+    spec = synth.SPECS[name]
+    keep, steps, warmup, peak_kind = EXTRA_WORKLOADS[name]
+    w = synth.make_workload(name, seed=rank, device=dev)
+    senders = [(s_.K, s_.V) for s_ in w.senders]
+    queries = [w.queries[s_.task] for s_ in w.senders]
+    c = cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads, spec.shape.head_dim,
+                     spec.m, max(spec.T), len(senders))
+    f = cb.Filter(c, senders, queries, keep, device=dev)
+    stream = torch.cuda.Stream(dev)
+    for _ in range(warmup):
+        f.run(stream)
+    c.sync_status(stream)
+    c.enable_stage_timing(2)
+    c.stage_times()
+    graph = None
+    if use_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for _ in range(steps):
+                f.run(stream)
+        for _ in range(2):
+            graph.replay()
+        torch.cuda.synchronize(dev)
+    sampler = ClockSampler(dev.index or 0)
+    sampler.start()
+    time.sleep(0.15)
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    t_wall0 = time.time()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    if graph is not None:
+        with torch.cuda.stream(stream):
+            graph.replay()
+    else:
+        for _ in range(steps):
+            f.run(stream)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    barrier(ws)
+    sampler.stop()
+    c.sync_status(stream)
+    timed_ms, timed_calls = c.stage_times()
+    graph = None
+    c.enable_stage_timing(False)
+    ms = max_over_ranks(ws, e0.elapsed_time(e1))
+    step_s = ms / steps / 1e3
+    accum = timed_ms["normalised_accumulation"] / max(1, timed_calls)
+    hbm_peak, tc_burst, tc_sus, src = peaks()
+    tc_peak = tc_sus if peak_kind == "sustained" else tc_burst
+    tot_b, score_b, compact_b, flops = workload_bytes_flops(spec, keep)
+    tokens = sum(f.Ts)
+    res = {"value": tokens * ws * steps / (ms / 1e3), "unit": UNIT, "ms_per_step": ms / steps, "steps": steps,
+           "warmup": warmup, "config": workload_config(spec, keep, 0, ws),
+           "hbm_gbs": tot_b / step_s / 1e9, "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
+           "algorithmic_bytes_per_step": tot_b,
+           "roofline": {"bound": "tensor", "kernel": "k_accum_tc", "duration_ms": accum,
+                        "achieved": flops / 2 / (accum / 1e3) / 1e12, "peak": tc_peak, "unit": "TFLOP/s",
+                        "frac": flops / 2 / (accum / 1e3) / 1e12 / tc_peak,
+                        "peak_source": "%s bf16 %s (cuBLAS)" % (src, peak_kind),
+                        "algorithmic_flops_per_launch": flops / 2},
+           "roofline_step": {"t_hbm_us": tot_b / (hbm_peak * 1e9) * 1e6,
+                             "t_tensor_us": flops / (tc_peak * 1e12) * 1e6,
+                             "frac": max(tot_b / (hbm_peak * 1e9), flops / (tc_peak * 1e12)) / step_s},
+           "score_kernels": {2: "tcgen05", 1: "mma.sync"}.get(c.score_path(), "none"),
+           "clocks": sampler.summary(t_wall0, t_wall1)}
+    del f, c, w, senders, queries
+    torch.cuda.empty_cache()
+    return res
 
 
 def run_ours(args):
@@ -636,17 +743,10 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.workload, "senders": len(senders), "T": list(spec.T[:3]), "m": spec.m,
-                   "n_layers": spec.shape.n_layers, "q_heads": spec.shape.n_q_heads,
-                   "kv_heads": spec.shape.n_kv_heads, "head_dim": spec.shape.head_dim, "keep": keep,
-                   "l2": "inputs larger than L2 (K+V %.2f GB per rank), no flush" % (
-                       sum(K.numel() * 4 for K, _ in inputs) / 1e9),
-                   "sender_states": len(inputs),
-                   "layout": ("paged: %d positions per page, pages in a random order" % args.paged)
-                             if args.paged else "strided [nL][Hkv][T][d]",
-                   "parallelism": "replicas" if ws > 1 else "single",
-                   "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential",
-                   "launch": launch_mode},
+        "config": workload_config(spec, keep, args.paged, ws),
+        "run": {"sender_states": len(inputs),
+                "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential",
+                "launch": launch_mode},
         "hbm_gbs": tot_b / step_s / 1e9,
         "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
         "hbm_frac_nominal": tot_b / step_s / 1e9 / 7900.0,   # of the 7.9 TB/s datasheet figure
@@ -687,10 +787,17 @@ def run_ours(args):
         out["e2e"] = e2e
     if pipelined:
         out["pipelined"] = pipelined
+    extra = [x for x in (args.workloads or "").split(",") if x]
+    if extra and not args.paged:
+        del f, c, w, senders, queries, states, states_all, inputs
+        torch.cuda.empty_cache()
+        out["workloads"] = {}
+        for name in extra:
+            out["workloads"][name] = time_workload(name, ws, rank, dev, not args.no_graph)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        out["cpu_baseline"] = oracle_sample(args.workload, args.cpu_layers)
+        out["cpu_baseline"] = oracle_sample(args.workload, args.cpu_layers, keep=keep)
     if rank == 0:
         print(json.dumps(out))
     if ws > 1:
@@ -714,9 +821,14 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=0, help="oracle layers per sample (0: by workload size)")
     ap.add_argument("--paged", type=int, default=0,
                     help="hold each sender cache in pages of this many positions (random page order)")
+    ap.add_argument("--workloads", default=None,
+                    help="comma-separated workloads timed after the headline and reported under 'workloads' "
+                         "(default: fanin,hybrid,sweep for the qwen8b headline, none otherwise; '' for none)")
     ap.add_argument("--wave", type=int, default=None,
                     help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()
+    if args.workloads is None:
+        args.workloads = ",".join(EXTRA_WORKLOADS) if args.workload == "qwen8b" else ""
     if args.impl == "reference":
         return run_reference(args)
     from paper_2609_32046_gb300.build import build, up_to_date, LIB_PATH
