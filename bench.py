@@ -505,6 +505,8 @@ def run_ours(args):
     states_all = list(states)
     c = cb.CacheBack(spec.shape.n_layers, spec.shape.n_q_heads, spec.shape.n_kv_heads, spec.shape.head_dim,
                      spec.m, max(spec.T), len(senders))
+    if args.score_sms:
+        c.set_score_sms(args.score_sms)
     if args.paged:
         # the same caches in a vLLM-style paged layout: pages of args.paged positions in a random order
         pk = {K.data_ptr(): paged_cache(cb, K, V, args.paged, seed=rank) for K, V in states}
@@ -746,6 +748,7 @@ def run_ours(args):
         "config": workload_config(spec, keep, args.paged, ws),
         "run": {"sender_states": len(inputs),
                 "schedule": ("waves of %d senders on two streams" % wave) if wave else "sequential",
+                "score_sms": args.score_sms or None,
                 "launch": launch_mode},
         "hbm_gbs": tot_b / step_s / 1e9,
         "hbm_frac": tot_b / step_s / 1e9 / hbm_peak,
@@ -824,6 +827,9 @@ def main():
     ap.add_argument("--workloads", default=None,
                     help="comma-separated workloads timed after the headline and reported under 'workloads' "
                          "(default: fanin,hybrid,sweep for the qwen8b headline, none otherwise; '' for none)")
+    ap.add_argument("--score-sms", type=int, default=0,
+                    help="SMs the persistent score kernels occupy (0: all); the rest run the previous "
+                         "wave's selection and compaction")
     ap.add_argument("--wave", type=int, default=None,
                     help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()

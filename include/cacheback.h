@@ -288,6 +288,18 @@ cb_status cb_stage_times(cb_ctx *ctx, float *ms, int32_t *calls);
  */
 cb_status cb_set_wait_limit(cb_ctx *ctx, int64_t limit_ns, int32_t stall_next_score);
 
+/*
+ * SMs the score kernels occupy (a runtime control; the paper has no counterpart).  The
+ * tcgen05 passes run one persistent CTA per SM on at most n_sms SMs (0, the default: every SM
+ * of the device), leaving the other SMs free for work on other streams: a batch's cb_select and
+ * cb_compact queued beside the next batch's cb_score run there (their blocks cannot share an SM
+ * with a score CTA), so selection and compaction of one wave of senders overlap the scoring of
+ * the next.  Scores, indices and messages do not depend on it (every sum keeps its order).
+ * The mma.sync passes ignore it.
+ * Errors: CB_EINVAL (NULL ctx, n_sms < 0).  Host-only; affects later calls.
+ */
+cb_status cb_set_score_sms(cb_ctx *ctx, int32_t n_sms);
+
 /* Free the context's scratch (after synchronising its device).  NULL is ignored. */
 void cb_destroy(cb_ctx *ctx);
 

@@ -22,7 +22,7 @@ STATUS_NAMES = ["CB_OK", "CB_EINVAL", "CB_ESHAPE", "CB_EBUDGET", "CB_ENOMEM", "C
 EXPORTED = ["cb_config_init", "cb_create", "cb_score", "cb_budget", "cb_select", "cb_compact",
             "cb_sync_status", "cb_destroy", "cb_last_error", "cb_scratch_bytes", "cb_score_path", "cb_select_noalloc",
             "cb_select_noalloc_status", "cb_gather", "cb_chain_budget", "cb_compact_rope",
-            "cb_enable_stage_timing", "cb_stage_times", "cb_set_wait_limit"]
+            "cb_enable_stage_timing", "cb_stage_times", "cb_set_wait_limit", "cb_set_score_sms"]
 
 
 class CBError(RuntimeError):
@@ -104,6 +104,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.cb_select_noalloc.restype = ctypes.c_int
     lib.cb_set_wait_limit.argtypes = [P, ctypes.c_int64, ctypes.c_int32]
     lib.cb_set_wait_limit.restype = ctypes.c_int
+    lib.cb_set_score_sms.argtypes = [P, ctypes.c_int32]
+    lib.cb_set_score_sms.restype = ctypes.c_int
     lib.cb_select_noalloc_status.argtypes = [P]
     lib.cb_select_noalloc_status.restype = ctypes.c_int
     lib.cb_enable_stage_timing.argtypes = [P, ctypes.c_int32]
@@ -336,6 +338,10 @@ class CacheBack:
         """cb_set_wait_limit: limit of one bounded device wait (0: the 1 s default); with
         stall_next_score the next tcgen05 cb_score makes one wait run out (failure-detection test)."""
         self._check(self.lib.cb_set_wait_limit(self.h, int(limit_ns), 1 if stall_next_score else 0))
+
+    def set_score_sms(self, n_sms: int = 0):
+        """cb_set_score_sms: SMs the persistent score kernels occupy (0: all)."""
+        self._check(self.lib.cb_set_score_sms(self.h, int(n_sms)))
 
     STAGES = ("row_statistics", "statistics_combine", "normalised_accumulation", "finalize")
 

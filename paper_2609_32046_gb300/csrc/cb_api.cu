@@ -74,6 +74,7 @@ struct cb_ctx {
     int32_t score_path = 0;         // kernels of the last cb_score: 2 tcgen05, 1 mma.sync, 0 none yet
     int64_t wait_ns = kDefaultWaitNs;   // limit of one bounded device wait (tcgen05 passes)
     int32_t stall_next = 0;         // failure-detection test: stall the next cb_score once
+    int32_t score_sms = 0;          // SMs of the persistent score kernels (0: all)
     cbk::StageTimer* timer = nullptr;
     std::string last_error;
 };
@@ -448,7 +449,8 @@ cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query*
             d.blk2_begin = b2; b2 += (int64_t)nS * d.n_chunk2;
         }
         int path = 0;
-        cudaError_t e = cbk::launch_score(*bt, strm, ctx->num_sms, &path);
+        const int sms = ctx->score_sms > 0 && ctx->score_sms < ctx->num_sms ? ctx->score_sms : ctx->num_sms;
+        cudaError_t e = cbk::launch_score(*bt, strm, sms, &path);
         ctx->score_path = path;
         delete bt;
         if (e != cudaSuccess) return fail(ctx, CB_ECUDA, "score launch failed: %s", cudaGetErrorString(e));
@@ -467,6 +469,14 @@ cb_status cb_set_wait_limit(cb_ctx* ctx, int64_t limit_ns, int32_t stall_next_sc
         return fail(ctx, CB_EINVAL, "stall_next_score must be 0 or 1");
     ctx->wait_ns = limit_ns ? limit_ns : kDefaultWaitNs;
     ctx->stall_next = stall_next_score;
+    return CB_OK;
+}
+
+cb_status cb_set_score_sms(cb_ctx* ctx, int32_t n_sms) {
+    if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
+    ctx->last_error.clear();
+    if (n_sms < 0) return fail(ctx, CB_EINVAL, "n_sms = %d must be >= 0", n_sms);
+    ctx->score_sms = n_sms;
     return CB_OK;
 }
 

@@ -266,6 +266,32 @@ def test_wave_schedule_matches_sequential():
 
 
 
+def test_results_do_not_depend_on_the_score_sms():
+    """cb_set_score_sms: the tcgen05 passes on fewer SMs (a smaller persistent grid, so other
+    contiguous work ranges) give the same bytes, and the wave schedule beside it too."""
+    name, shape, Ts, m, keep, extra = [c for c in CASES if c[0] == "forty_senders"][0]
+    w = _workload(name, shape, Ts, m)
+    pairs = [(s.K.cuda(), s.V.cuda()) for s in w.senders]
+    qs = [w.queries[s.task].cuda() for s in w.senders]
+    c = make_cb(w.spec.shape, max(Ts), m, len(Ts), score_kernel=2)
+    ref = cb.Filter(c, pairs, qs, keep).run()
+    c.sync_status()
+    for n_sms in (97, 16, 1):
+        c.set_score_sms(n_sms)
+        got = cb.Filter(c, pairs, qs, keep).run(wave=9)
+        c.sync_status()
+        assert c.score_path() == 2
+        for a, b in zip(ref.scores, got.scores):
+            assert torch.equal(a.view(torch.int32), b.view(torch.int32)), n_sms
+        for a, b, B in zip(ref.idx, got.idx, ref.budgets):
+            assert torch.equal(a[:B], b[:B]), n_sms
+        assert torch.equal(ref.k_out.view(torch.int16), got.k_out.view(torch.int16)), n_sms
+        assert torch.equal(ref.v_out.view(torch.int16), got.v_out.view(torch.int16)), n_sms
+    c.set_score_sms(0)
+    with pytest.raises(cb.CBError):
+        c.set_score_sms(-1)
+
+
 @pytest.mark.parametrize("kernel", [1, 2], ids=["mma_sync", "tcgen05"])
 @pytest.mark.parametrize("scale", [70.0, 150.0], ids=["large_finite", "overflowing"])
 def test_extreme_logit_rows(kernel, scale):
