@@ -489,11 +489,25 @@ def time_workload(name: str, ws: int, rank: int, dev, use_graph: bool):
     return res
 
 
+def layer_subset(name: str, layers: int):
+    """The workload's spec with only its first `layers` layers (0: unchanged), registered under a
+    name of its own so that the inputs are generated for that shape."""
+    import dataclasses
+    import synth
+    spec = synth.SPECS[name]
+    if layers <= 0 or layers >= spec.shape.n_layers:
+        return name
+    sub = "%s_l%d" % (name, layers)
+    synth.SPECS[sub] = dataclasses.replace(spec, name=sub, shape=dataclasses.replace(spec.shape, n_layers=layers))
+    return sub
+
+
 def run_ours(args):
     import torch
     import paper_2609_32046_gb300 as cb
     import synth
     ws, rank, local = dist_init()
+    args.workload = layer_subset(args.workload, args.layers)
     spec = synth.SPECS[args.workload]
     keep = args.keep if args.keep is not None else spec.keeps[0]
     dev = torch.device("cuda", local)
@@ -827,12 +841,17 @@ def main():
     ap.add_argument("--workloads", default=None,
                     help="comma-separated workloads timed after the headline and reported under 'workloads' "
                          "(default: fanin,hybrid,sweep for the qwen8b headline, none otherwise; '' for none)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="score only the first N layers of the workload's shape (a smaller case of the same "
+                         "kernels, e.g. for an ncu capture); 0: all")
     ap.add_argument("--score-sms", type=int, default=0,
                     help="SMs the persistent score kernels occupy (0: all); the rest run the previous "
                          "wave's selection and compaction")
     ap.add_argument("--wave", type=int, default=None,
                     help="senders per wave of the two-stream schedule (default 0: sequential)")
     args = ap.parse_args()
+    if args.layers and args.workloads is None:
+        args.workloads = ""
     if args.workloads is None:
         args.workloads = ",".join(EXTRA_WORKLOADS) if args.workload == "qwen8b" else ""
     if args.impl == "reference":
