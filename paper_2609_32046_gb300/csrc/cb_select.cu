@@ -90,11 +90,16 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     __shared__ float red[32];
     __shared__ float head[kMaxSpanWidth];   // scores of the first span
     __shared__ int64_t sel_bucket, sel_before;
+    __shared__ int64_t part_j;      // the span taken in part, when its run is found by a warp
+    __shared__ int32_t part_take;
 
     // this block's sender in shared memory: reads of the parameter array at a run-time index
     // are slow, and with 64 registers a thread the compiler re-reads such values in loops
     __shared__ SelectSender sd;
-    if (threadIdx.x == 0) sd = bt.s[blockIdx.x];
+    if (threadIdx.x == 0) {
+        sd = bt.s[blockIdx.x];
+        part_j = -1;
+    }
     __syncthreads();
     const int64_t T = sd.T, B = sd.B;
     const int w = bt.span_w;
@@ -114,14 +119,45 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     const bool sink = bt.n_sink > 0;
     const int64_t tile = (int64_t)(kScoreTile / w) * w;     // whole spans per tile
     const int64_t ntile = (T + tile - 1) / tile;
+    // width-16 spans, one a thread: each thread reads its span's scores with four 16-byte loads
+    // (scores are 16-byte aligned) and sums them in index order, with no staging
+    const bool direct = w == 16 && nsp <= kSelThreads;
+    float mx = -INFINITY;
+    if (direct && tid < nsp) {
+        const int64_t lo = (int64_t)tid * 16;
+        const int n = (int)(T - lo < 16 ? T - lo : 16);
+        float v[16];
+        if (n == 16) {
+            const float4* p = reinterpret_cast<const float4*>(S + lo);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float4 x = p[q];
+                v[4 * q] = x.x;
+                v[4 * q + 1] = x.y;
+                v[4 * q + 2] = x.z;
+                v[4 * q + 3] = x.w;
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < 16; ++k) v[k] = k < n ? S[lo + k] : 0.f;
+        }
+        float acc = 0.f;
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+            if (k < n) {
+                mx = fmaxf(mx, v[k]);
+                acc += v[k];
+                if (tid == 0) head[k] = v[k];
+            }
+        if (!(tid == 0 && sink)) keys[tid] = __fdiv_rn(acc, (float)n);
+    }
     float nxt[kPerThread];
 #pragma unroll
     for (int q = 0; q < kPerThread; ++q) {
         const int k = tid + q * kSelThreads;
-        nxt[q] = k < tile && k < T ? S[k] : 0.f;
+        nxt[q] = !direct && k < tile && k < T ? S[k] : 0.f;
     }
-    float mx = -INFINITY;
-    for (int64_t it = 0; it < ntile; ++it) {
+    for (int64_t it = 0; it < (direct ? 0 : ntile); ++it) {
         const int64_t t0 = it * tile, n = T - t0 < tile ? T - t0 : tile;
         float* ts = dsm + (it & 1) * kPadTile;
 #pragma unroll
@@ -170,11 +206,17 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
         keys[0] = __fdiv_rn(acc, (float)hi);
     }
     // a single tile still holds every score (the partial span's best position is looked up there)
-    const float* all_s = ntile == 1 ? dsm : nullptr;
+    const float* all_s = ntile == 1 && !direct ? dsm : nullptr;
     const int64_t need = B - F.count(0, T);
     __syncthreads();
 
     // 2. weighted radix select of the threshold key
+    uint32_t my_key = 0u, my_u = 0u;   // with one span a thread: its key and unforced positions
+    if (direct && tid < nsp) {
+        const int64_t lo = (int64_t)tid * w, hi = lo + w < T ? lo + w : T;
+        my_key = order_key(keys[tid]);
+        my_u = (uint32_t)((hi - lo) - F.count(lo, hi));
+    }
     uint32_t prefix = 0u, pmask = 0u;
     int64_t rem = need;
     if (need > 0) {
@@ -182,12 +224,17 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             const int shift = 24 - 8 * pass;
             if (tid < 256) hist[tid] = 0u;
             __syncthreads();
-            for (int64_t j = tid; j < nsp; j += kSelThreads) {
-                const uint32_t key = order_key(keys[j]);
-                if ((key & pmask) != prefix) continue;
-                const int64_t lo = j * w, hi = lo + w < T ? lo + w : T;
-                const uint32_t u = (uint32_t)((hi - lo) - F.count(lo, hi));
-                if (u) atomicAdd(&hist[(key >> shift) & 255u], u);
+            if (direct) {
+                // one span a thread: its key and unforced count were found once, before the passes
+                if (my_u && (my_key & pmask) == prefix) atomicAdd(&hist[(my_key >> shift) & 255u], my_u);
+            } else {
+                for (int64_t j = tid; j < nsp; j += kSelThreads) {
+                    const uint32_t key = order_key(keys[j]);
+                    if ((key & pmask) != prefix) continue;
+                    const int64_t lo = j * w, hi = lo + w < T ? lo + w : T;
+                    const uint32_t u = (uint32_t)((hi - lo) - F.count(lo, hi));
+                    if (u) atomicAdd(&hist[(key >> shift) & 255u], u);
+                }
             }
             __syncthreads();
             if (warp == 0) {
@@ -285,6 +332,9 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             if (take == u) {
                 left = lo;
                 right = hi - 1;
+            } else if (take > 0 && coop && w <= 32) {
+                part_j = j;                // its run is found by a warp below (at most one such span)
+                part_take = (int32_t)take;
             } else if (take > 0) {
                 // highest-scoring unforced position (lowest index on ties)
                 int64_t c = -1;
@@ -330,6 +380,28 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     }
     if (coop) {
         __syncthreads();
+        if (part_j >= 0 && warp == 0) {
+            // the partial span's take unforced positions nearest its highest-scoring unforced one
+            // (lowest index on ties), distance ties to the lower index: ranked by (distance, index)
+            const int64_t j = part_j, lo = j * w, hi = lo + w < T ? lo + w : T;
+            const int64_t t = lo + lane;
+            const bool unf = t < hi && !F.at(t);
+            const float v = unf ? S[t] : -INFINITY;
+            float vm = v;
+#pragma unroll
+            for (int o = 16; o; o >>= 1) vm = fmaxf(vm, __shfl_xor_sync(0xffffffffu, vm, o));
+            const int cl = __ffs(__ballot_sync(0xffffffffu, unf && v == vm)) - 1;
+            const int d = unf ? abs(lane - cl) : (1 << 20);
+            int rank = 0;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+                const int dk = __shfl_sync(0xffffffffu, d, k);
+                rank += (dk < d || (dk == d && k < lane)) ? 1 : 0;
+            }
+            const unsigned sel = __ballot_sync(0xffffffffu, unf && rank < part_take);
+            if (lane == 0) span_run[j] = (int32_t)((__ffs(sel)) | ((32 - __clz(sel)) << 16));
+        }
+        __syncthreads();
         // 32-bit arithmetic throughout (T < 2^31): this loop is bound by instruction issue
         const int32_t T32 = (int32_t)T, B32 = (int32_t)(B < T ? B : T), fa = (int32_t)F.a, fb = (int32_t)F.b;
         const int32_t nsp32 = (int32_t)nsp;
@@ -339,6 +411,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             const int32_t lo = j * w, hi = lo + w < T32 ? lo + w : T32;
             const int32_t run = span_run[j];
             const int32_t left = lo + (run & 0xffff) - 1, right = lo + (run >> 16) - 1;
+            if (right < left && lo >= fa && hi <= fb) continue;   // nothing of this span is kept
             int32_t base = span_at[j];
             for (int32_t c0 = lo; c0 < hi; c0 += 32) {
                 const int32_t t = c0 + lane;
