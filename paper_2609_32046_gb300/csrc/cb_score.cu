@@ -248,22 +248,27 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
 // ---------------------------------------------------------------------------
 // combine: per-row log2 offset = max + log2(sum) + log2(G) over all chunks
 // ---------------------------------------------------------------------------
-// Thread = row of one (sender, group s).  Its partial slots are merged as four chains
-// (slots j, j + 4, j + 8, ... for j = 0..3, each with an online max / sum in slot order), then
-// the four chain results in chain order: a fixed order, so the offsets are deterministic.  All
-// slots of a batch of 32 are loaded before any is merged (the partials mostly come from DRAM),
-// and one thread a row keeps the whole grid in one wave.
-constexpr int kCombRows = 256;     // rows (threads) per block
-constexpr int kCombBatch = 32;     // slots loaded before they are merged
-__global__ void __launch_bounds__(kCombRows) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
+// A row of one (sender, group s) merges its partial slots as four chains (slots j, j + 4, j + 8,
+// ... for j = 0..3, each with an online max / sum in slot order), then the four chain results in
+// chain order: a fixed order, so the offsets are deterministic and the same for both layouts.
+// TPR = 1: one thread a row merges all four chains (many rows: the grid then fits in one wave);
+// TPR = 4: four threads a row, one a chain, exchanging their results by shuffles (few rows with
+// many slots each, e.g. long senders: four times the threads in flight).  A batch of slots is
+// loaded before any is merged (the partials mostly come from DRAM).
+constexpr int kCombThreads = 256;
+constexpr int kCombBatch = 32;     // slots of a row loaded before they are merged
+template <int TPR>
+__global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
+    constexpr int RPB = kCombThreads / TPR;   // rows per block
+    constexpr int NC = 4 / TPR;               // chains a thread merges
     const int nS = bt.n_layers * bt.n_kv_heads;
     int i = 0;
     int64_t blk = blockIdx.x;
-    // blocks are laid out sender by sender, nS * ceil(rows / 256) of them per sender
+    // blocks are laid out sender by sender, nS * ceil(rows / RPB) of them per sender
     for (; i < bt.n; ++i) {
         const int R_i = bt.s[i].m * G;
         const int rows_i = bt.ext ? (int)rows_pad128(R_i) : R_i;
-        const int64_t nb = (int64_t)nS * ((rows_i + kCombRows - 1) / kCombRows);
+        const int64_t nb = (int64_t)nS * ((rows_i + RPB - 1) / RPB);
         if (blk < nb) break;
         blk -= nb;
     }
@@ -271,10 +276,12 @@ __global__ void __launch_bounds__(kCombRows) k_combine(const __grid_constant__ S
     const ScoreSender& sd = bt.s[i];
     const int R = sd.m * G;
     const int rows = bt.ext ? (int)rows_pad128(R) : R;
-    const int nrb = (rows + kCombRows - 1) / kCombRows;
+    const int nrb = (rows + RPB - 1) / RPB;
     const int s = (int)(blk / nrb);
-    const int row = (int)(blk % nrb) * kCombRows + threadIdx.x;
-    if (row >= rows) return;
+    const int row = (int)(blk % nrb) * RPB + (int)threadIdx.x / TPR;
+    const int c0l = TPR == 1 ? 0 : (int)threadIdx.x % TPR;   // the thread's first chain
+    if (row >= rows) return;                                   // (the four threads of a row together)
+    const unsigned gmask = TPR == 1 ? 0u : 0xFu << ((threadIdx.x & 31) & ~3u);
     const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
     const int r_tok = row / G, hh = row - r_tok * G;
     const uint16_t* qrow = sd.q + (int64_t)l * sd.qs_l + (int64_t)r_tok * sd.qs_t + (int64_t)(g * G + hh) * sd.qs_h;
@@ -304,34 +311,37 @@ __global__ void __launch_bounds__(kCombRows) k_combine(const __grid_constant__ S
     };
     // the query tokens' own keys: row (token r, head h) also attends to query keys 0..r, key u
     // on chain u mod 4 (each chain in increasing u); logits in the statistics' log2 domain
-    auto merge_self_keys = [&](float (&M)[4], float (&L)[4]) {
+    auto merge_self_keys = [&](float (&M)[NC], float (&L)[NC]) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-            for (int u = j; u <= r_tok; u += 4)
+        for (int k = 0; k < NC; ++k)
+            for (int u = c0l + k; u <= r_tok; u += 4)
                 merge_logit(dot_row(sd.kself + (int64_t)l * sd.kss_l + (int64_t)u * sd.kss_t + (int64_t)g * sd.kss_h) *
-                                bt.scale_log2e, M[j], L[j]);
+                                bt.scale_log2e, M[k], L[k]);
     };
     float off = 0.f;
     if (row < R) {
-        float M[4], L[4];
+        float M[NC], L[NC];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) { M[j] = -INFINITY; L[j] = 0.f; }
+        for (int k = 0; k < NC; ++k) { M[k] = -INFINITY; L[k] = 0.f; }
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
-        for (int c0 = 0; c0 < sd.n_chunk1; c0 += kCombBatch) {
-            float2 vv[kCombBatch];
+        for (int cb = 0; cb < sd.n_chunk1; cb += kCombBatch) {
+            constexpr int NL = kCombBatch / TPR;   // this thread's slots of the batch
+            float2 vv[NL];
 #pragma unroll
-            for (int q = 0; q < kCombBatch; ++q)
-                vv[q] = c0 + q < sd.n_chunk1 ? st[(int64_t)(c0 + q) * R] : make_float2(-INFINITY, 0.f);
+            for (int q = 0; q < NL; ++q) {
+                const int c = cb + (TPR == 1 ? q : 4 * q + c0l);   // chain c mod 4 (cb a multiple of 32)
+                vv[q] = c < sd.n_chunk1 ? st[(int64_t)c * R] : make_float2(-INFINITY, 0.f);
+            }
 #pragma unroll
-            for (int q = 0; q < kCombBatch; ++q) {
+            for (int q = 0; q < NL; ++q) {
                 const float2 v = vv[q];
-                const int j = q & 3;   // slot c0 + q is on chain (c0 + q) mod 4, c0 a multiple of 32
+                const int k = TPR == 1 ? (q & 3) : 0;
                 if (v.x == -INFINITY) continue;
-                if (v.x > M[j]) {
-                    L[j] = (M[j] == -INFINITY ? 0.f : L[j] * ex2(M[j] - v.x)) + v.y;
-                    M[j] = v.x;
+                if (v.x > M[k]) {
+                    L[k] = (M[k] == -INFINITY ? 0.f : L[k] * ex2(M[k] - v.x)) + v.y;
+                    M[k] = v.x;
                 } else {
-                    L[j] += v.y * ex2(v.x - M[j]);
+                    L[k] += v.y * ex2(v.x - M[k]);
                 }
             }
         }
@@ -340,28 +350,49 @@ __global__ void __launch_bounds__(kCombRows) k_combine(const __grid_constant__ S
         // tensor-memory path offsets each chunk by the maximum of its first 32 logits, so a logit
         // far larger later in the chunk overflows exp2).  Such rows, rare, are recomputed here
         // from Q and K directly: position t on chain t mod 4.
-        if (!(L[0] <= FLT_MAX) || !(L[1] <= FLT_MAX) || !(L[2] <= FLT_MAX) || !(L[3] <= FLT_MAX)) {
+        bool bad = false;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) { M[j] = -INFINITY; L[j] = 0.f; }
+        for (int k = 0; k < NC; ++k) bad = bad || !(L[k] <= FLT_MAX);
+        if (TPR == 4) {
+            bad = __shfl_xor_sync(gmask, (int)bad, 1) != 0 || bad;
+            bad = __shfl_xor_sync(gmask, (int)bad, 2) != 0 || bad;
+        }
+        if (bad) {
+#pragma unroll
+            for (int k = 0; k < NC; ++k) { M[k] = -INFINITY; L[k] = 0.f; }
             const uint16_t* kbase = sd.k + (int64_t)l * sd.ks_l + (int64_t)g * sd.ks_h;
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-                for (int64_t t = j; t < sd.T; t += 4) {
+            for (int k = 0; k < NC; ++k)
+                for (int64_t t = c0l + k; t < sd.T; t += 4) {
                     const int64_t ro = row_offset(sd.pm, sd.ks_p, t);
-                    merge_logit(ro < 0 ? 0.f : dot_row(kbase + ro) * bt.scale_log2e, M[j], L[j]);   // a bad page reads as zeros
+                    merge_logit(ro < 0 ? 0.f : dot_row(kbase + ro) * bt.scale_log2e, M[k], L[k]);   // a bad page reads as zeros
                 }
             if (sd.kself) merge_self_keys(M, L);
         }
+        // the four chains in chain order
+        float Mc[4], Lc[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (TPR == 1) {
+                Mc[k] = M[k];
+                Lc[k] = L[k];
+            } else {
+                const int src = ((int)threadIdx.x & 31 & ~3) + k;
+                Mc[k] = __shfl_sync(gmask, M[0], src);
+                Lc[k] = __shfl_sync(gmask, L[0], src);
+            }
+        }
         float Mx = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) Mx = fmaxf(Mx, M[k]);
+        for (int k = 0; k < 4; ++k) Mx = fmaxf(Mx, Mc[k]);
         float Lx = 0.f;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-            if (M[k] != -INFINITY) Lx += L[k] * ex2(M[k] - Mx);
+            if (Mc[k] != -INFINITY) Lx += Lc[k] * ex2(Mc[k] - Mx);
         off = Mx + log2f(Lx) + log2f((float)G);
-        bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
+        if (c0l == 0) bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
     }
+    if (c0l != 0) return;
     if (bt.ext) {
         // the tcgen05 pass 2 adds -off / scale_log2e to the logit inside the contraction
         // (one more K-step against a column of ones): three bf16 terms carry it to ~24 bits
@@ -639,22 +670,36 @@ cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-int64_t combine_blocks(const ScoreBatch& b) {
+// Rows of all senders of a batch; few rows (long senders, few groups) take four threads a row.
+int64_t combine_rows(const ScoreBatch& b) {
     const int G = b.n_q_heads / b.n_kv_heads;
     const int64_t nS = (int64_t)b.n_layers * b.n_kv_heads;
+    int64_t rows = 0;
+    for (int i = 0; i < b.n; ++i) {
+        const int64_t R = (int64_t)b.s[i].m * G;
+        rows += nS * (b.ext ? rows_pad128(R) : R);
+    }
+    return rows;
+}
+
+template <int TPR>
+cudaError_t launch_combine_t(const ScoreBatch& b, cudaStream_t st) {
+    const int G = b.n_q_heads / b.n_kv_heads;
+    const int64_t nS = (int64_t)b.n_layers * b.n_kv_heads;
+    constexpr int RPB = kCombThreads / TPR;
     int64_t nb = 0;
     for (int i = 0; i < b.n; ++i) {
         const int64_t R = (int64_t)b.s[i].m * G;
         const int64_t rows = b.ext ? rows_pad128(R) : R;
-        nb += nS * ((rows + kCombRows - 1) / kCombRows);
+        nb += nS * ((rows + RPB - 1) / RPB);
     }
-    return nb;
+    k_combine<TPR><<<(unsigned)nb, kCombThreads, 0, st>>>(b, G);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_combine(const ScoreBatch& b, cudaStream_t st) {
-    const int G = b.n_q_heads / b.n_kv_heads;
-    k_combine<<<(unsigned)combine_blocks(b), kCombRows, 0, st>>>(b, G);
-    return cudaGetLastError();
+    // four threads a row while that stays well within one wave of resident threads
+    return combine_rows(b) <= 40000 ? launch_combine_t<4>(b, st) : launch_combine_t<1>(b, st);
 }
 
 
@@ -683,7 +728,7 @@ cudaError_t launch_dg(const ScoreBatch& b, cudaStream_t st) {
     stage_mark(b.timer, kStageStart, st);
     k_stats<D, G><<<(unsigned)nblk1, kThreads, smem1, st>>>(b);
     stage_mark(b.timer, kStageStats, st);
-    k_combine<<<(unsigned)combine_blocks(b), kCombRows, 0, st>>>(b, G);
+    launch_combine(b, st);
     stage_mark(b.timer, kStageCombine, st);
     k_accum<D, G><<<(unsigned)nblk2, kThreads, smem2, st>>>(b);
     stage_mark(b.timer, kStageAccum, st);

@@ -36,6 +36,7 @@ constexpr int kPerThread = kScoreTile / kSelThreads;    // scores each thread st
 constexpr int kSmemSpans = 8192;     // span means kept in shared memory when there are at most this many
 // two score tiles, the span means, and (one span a thread) each span's [left, right] run
 constexpr size_t kSelDynSmem = (size_t)(2 * kPadTile + kSmemSpans + kSelThreads) * sizeof(float);
+constexpr int kDirectPer = 4;        // width-16 spans a thread reads directly (up to 4096 spans)
 
 __device__ __forceinline__ int pad(int k) { return k + (k >> 5); }
 
@@ -119,12 +120,16 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     const bool sink = bt.n_sink > 0;
     const int64_t tile = (int64_t)(kScoreTile / w) * w;     // whole spans per tile
     const int64_t ntile = (T + tile - 1) / tile;
-    // width-16 spans, one a thread: each thread reads its span's scores with four 16-byte loads
-    // (scores are 16-byte aligned) and sums them in index order, with no staging
-    const bool direct = w == 16 && nsp <= kSelThreads;
+    // width-16 spans, up to four a thread (spans tid, tid + 1024, ...): each thread reads its
+    // spans' scores with four 16-byte loads each (scores are 16-byte aligned) and sums them in
+    // index order, with no staging
+    const bool direct = w == 16 && nsp <= (int64_t)kDirectPer * kSelThreads;
     float mx = -INFINITY;
-    if (direct && tid < nsp) {
-        const int64_t lo = (int64_t)tid * 16;
+#pragma unroll
+    for (int q8 = 0; q8 < kDirectPer; ++q8) {
+        const int64_t js = tid + (int64_t)q8 * kSelThreads;
+        if (!direct || js >= nsp) break;
+        const int64_t lo = js * 16;
         const int n = (int)(T - lo < 16 ? T - lo : 16);
         float v[16];
         if (n == 16) {
@@ -147,9 +152,9 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             if (k < n) {
                 mx = fmaxf(mx, v[k]);
                 acc += v[k];
-                if (tid == 0) head[k] = v[k];
+                if (js == 0) head[k] = v[k];
             }
-        if (!(tid == 0 && sink)) keys[tid] = __fdiv_rn(acc, (float)n);
+        if (!(js == 0 && sink)) keys[js] = __fdiv_rn(acc, (float)n);
     }
     float nxt[kPerThread];
 #pragma unroll
@@ -211,11 +216,17 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     __syncthreads();
 
     // 2. weighted radix select of the threshold key
-    uint32_t my_key = 0u, my_u = 0u;   // with one span a thread: its key and unforced positions
-    if (direct && tid < nsp) {
-        const int64_t lo = (int64_t)tid * w, hi = lo + w < T ? lo + w : T;
-        my_key = order_key(keys[tid]);
-        my_u = (uint32_t)((hi - lo) - F.count(lo, hi));
+    uint32_t my_key[kDirectPer], my_u[kDirectPer];   // direct: the thread's spans' keys and unforced positions
+#pragma unroll
+    for (int q8 = 0; q8 < kDirectPer; ++q8) {
+        const int64_t js = tid + (int64_t)q8 * kSelThreads;
+        my_key[q8] = 0u;
+        my_u[q8] = 0u;
+        if (direct && js < nsp) {
+            const int64_t lo = js * w, hi = lo + w < T ? lo + w : T;
+            my_key[q8] = order_key(keys[js]);
+            my_u[q8] = (uint32_t)((hi - lo) - F.count(lo, hi));
+        }
     }
     uint32_t prefix = 0u, pmask = 0u;
     int64_t rem = need;
@@ -225,8 +236,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
             if (tid < 256) hist[tid] = 0u;
             __syncthreads();
             if (direct) {
-                // one span a thread: its key and unforced count were found once, before the passes
-                if (my_u && (my_key & pmask) == prefix) atomicAdd(&hist[(my_key >> shift) & 255u], my_u);
+                // the thread's spans: their keys and unforced counts were found once, before the passes
+#pragma unroll
+                for (int q8 = 0; q8 < kDirectPer; ++q8)
+                    if (my_u[q8] && (my_key[q8] & pmask) == prefix)
+                        atomicAdd(&hist[(my_key[q8] >> shift) & 255u], my_u[q8]);
             } else {
                 for (int64_t j = tid; j < nsp; j += kSelThreads) {
                     const uint32_t key = order_key(keys[j]);
@@ -306,13 +320,14 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
 
     // 4. write positions in source order.  Each thread settles what its spans contribute:
     // everything, only the forced positions, or the forced ones plus the run [left, right]
-    // around the partial span's best position.  With one span a thread, a span's output start
-    // (in place of its mean, which is no longer needed) and its run go to shared memory and each
-    // warp then writes whole spans, 32 consecutive positions per step, so the stores are
-    // coalesced; with several (measured faster that way), every thread writes its own spans.
-    const bool coop = nsp <= kSelThreads;   // one span a thread (more: each thread writes its own)
+    // around the partial span's best position.  With one span a thread, or when the scores were
+    // read directly (the staging buffers then hold the runs), a span's output start (in place of
+    // its mean, which is no longer needed) and its run go to shared memory and each warp then
+    // writes whole spans, 32 consecutive positions per step, so the stores are coalesced;
+    // otherwise every thread writes its own spans.
+    const bool coop = nsp <= kSelThreads || direct;
     int32_t* span_at = reinterpret_cast<int32_t*>(keys);
-    int32_t* span_run = reinterpret_cast<int32_t*>(dsm + 2 * kPadTile + kSmemSpans);
+    int32_t* span_run = reinterpret_cast<int32_t*>(direct ? dsm : dsm + 2 * kPadTile + kSmemSpans);
     {
         int64_t tb = tie_before;
         for (int64_t j = j0; j < j1; ++j) {
