@@ -543,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_accum(const __grid_constant__ S
 // Block (64-position tile, sender); thread (slice k, quad q) sums slice k of the groups
 // (s = k, k + 16, ... in increasing order) for the four consecutive positions of quad q:
 // quads 2..17 are the tile (U, N and D), quads 0, 1 and 18, 19 the kHalo positions on each
-// side (U only, for Pool).  Nine groups' loads are issued before they are added (the partials
+// side (U only, for Pool).  A batch of groups' loads is issued before they are added (the partials
 // mostly come from DRAM, so the kernel needs many bytes in flight), with one 16-byte load per
 // quad where the sender's partial rows are 16-byte aligned.  The 16 slice sums of every
 // position are then added in slice order in shared memory, U is pooled and C and S written.
@@ -552,9 +552,12 @@ constexpr int kFinPos = 64;                          // output positions per blo
 constexpr int kFinQuads = kFinPos / 4 + kHalo / 2;   // 16 tile quads + 2 on each side
 constexpr int kFinSpan = 4 * kFinQuads;              // positions whose U is summed
 constexpr int kFinThreads = kFinSlices * kFinQuads;  // 320
-constexpr int kFinBatch = 9;                         // groups loaded before they are added
 
+// BATCH: groups of a slice loaded before they are added (9 for 288 groups; fewer groups, e.g. 64,
+// take a smaller batch, whose smaller register footprint fits several blocks an SM)
+template <int BATCH>
 __global__ void __launch_bounds__(kFinThreads) k_finalize(const __grid_constant__ ScoreBatch bt) {
+    constexpr int kFinBatch = BATCH;
     __shared__ float su[kFinSlices][kFinSpan];
     __shared__ float sn[kFinSlices][kFinPos];
     __shared__ float sdn[kFinSlices][kFinPos];
@@ -666,7 +669,11 @@ cudaError_t launch_finalize(const ScoreBatch& b, cudaStream_t st) {
     int64_t maxT = 0;
     for (int i = 0; i < b.n; ++i) maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
     dim3 grid((unsigned)((maxT + kFinPos - 1) / kFinPos), (unsigned)b.n);
-    k_finalize<<<grid, kFinThreads, 0, st>>>(b);
+    const int per_slice = (b.n_layers * b.n_kv_heads + kFinSlices - 1) / kFinSlices;
+    if (per_slice <= 4)
+        k_finalize<4><<<grid, kFinThreads, 0, st>>>(b);
+    else
+        k_finalize<9><<<grid, kFinThreads, 0, st>>>(b);
     return cudaGetLastError();
 }
 
