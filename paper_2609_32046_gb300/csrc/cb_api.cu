@@ -12,6 +12,7 @@
 #include <vector>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "cacheback.h"
 #include "cb_internal.cuh"
@@ -338,8 +339,17 @@ void cb_destroy(cb_ctx* ctx) {
     delete ctx;
 }
 
+namespace {
+// An NVTX range over one call of the C-ABI (header-only NVTX: free unless a profiler listens).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
+
 cb_status cb_score(cb_ctx* ctx, int32_t n, const cb_kv* senders, const cb_query* queries, float* const* scores,
                    void* stream) {
+    NvtxRange nr("cb_score");
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     ctx->last_error.clear();
     const cb_config& c = ctx->cfg;
@@ -482,6 +492,7 @@ cb_status cb_set_score_sms(cb_ctx* ctx, int32_t n_sms) {
 
 cb_status cb_select(cb_ctx* ctx, int32_t n, const float* const* scores, const int64_t* T, const int64_t* budget,
                     int32_t* const* idx, void* stream) {
+    NvtxRange nr("cb_select");
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     ctx->last_error.clear();
     const cb_config& c = ctx->cfg;
@@ -618,6 +629,7 @@ extern "C" {
 cb_status cb_compact(cb_ctx* ctx, int32_t n, const cb_kv* senders, const int32_t* const* idx, const int64_t* budget,
                      void* k_out, void* v_out, int64_t out_capacity, const int64_t* out_offset, int64_t o_layer,
                      int64_t o_head, void* stream) {
+    NvtxRange nr("cb_compact");
     return compact_impl(ctx, n, senders, idx, budget, k_out, v_out, out_capacity, out_offset, o_layer, o_head,
                         nullptr, stream);
 }
@@ -626,6 +638,7 @@ cb_status cb_compact_rope(cb_ctx* ctx, int32_t n, const cb_kv* senders, const in
                           const int64_t* budget, void* k_out, void* v_out, int64_t out_capacity,
                           const int64_t* out_offset, int64_t o_layer, int64_t o_head, double rope_base,
                           int32_t rope_style, int64_t pos0, void* stream) {
+    NvtxRange nr("cb_compact_rope");
     const RopeArgs r{rope_base, rope_style, pos0};
     return compact_impl(ctx, n, senders, idx, budget, k_out, v_out, out_capacity, out_offset, o_layer, o_head, &r,
                         stream);
@@ -677,6 +690,7 @@ cb_status cb_stage_times(cb_ctx* ctx, float* ms, int32_t* calls) {
 cb_status cb_gather(cb_ctx* ctx, int32_t n, const void* const* src, const int64_t* T, int64_t src_stride,
                     int64_t row_bytes, const int32_t* const* idx, const int64_t* count, void* out,
                     int64_t out_capacity, const int64_t* out_offset, int64_t out_stride, void* stream) {
+    NvtxRange nr("cb_gather");
     if (!ctx) return fail(nullptr, CB_EINVAL, "ctx is NULL");
     ctx->last_error.clear();
     if (n < 1) return fail(ctx, CB_ESHAPE, "n = %d < 1", n);
