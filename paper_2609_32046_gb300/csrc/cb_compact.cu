@@ -17,7 +17,7 @@ namespace cbk {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 2;
 
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
     uint4 v;
@@ -84,8 +84,10 @@ cudaError_t launch_compact(const CompactBatch& b, cudaStream_t st, int num_sms) 
     if (max_B == 0) return cudaSuccess;
     const int segs = 2 * b.n_layers * b.n_kv_heads;
     const int rows_per_pass = kThreads / (b.head_dim / 8);
-    // about 8 resident blocks per SM over the batch; each block walks its slice of rows
-    int64_t slices = ((int64_t)num_sms * 8 + (int64_t)segs * b.n - 1) / ((int64_t)segs * b.n);
+    // about 24 blocks per SM over the batch (three waves of eight resident blocks); each block
+    // walks its slice of rows (two loads in flight a thread over many blocks moved more bytes
+    // than four over fewer)
+    int64_t slices = ((int64_t)num_sms * 24) / ((int64_t)segs * b.n);
     const int64_t need = (max_B + (int64_t)rows_per_pass * kUnroll - 1) / ((int64_t)rows_per_pass * kUnroll);
     if (slices > need) slices = need;
     if (slices < 1) slices = 1;
