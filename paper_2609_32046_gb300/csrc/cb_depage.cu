@@ -77,8 +77,9 @@ cudaError_t launch_depage(const DepageBatch& b, cudaStream_t st, int num_sms) {
     int64_t maxT = 0;
     for (int i = 0; i < b.n; ++i) maxT = b.s[i].T > maxT ? b.s[i].T : maxT;
     const int64_t pieces = maxT * b.n_kv_heads * kPieces;
-    // about 8 resident blocks per SM over the whole grid
-    int64_t x = ((int64_t)num_sms * 8 + (int64_t)b.n * b.n_layers - 1) / ((int64_t)b.n * b.n_layers);
+    // about 48 blocks per SM over the whole grid (six waves of eight resident blocks): more,
+    // shorter blocks kept more of the copy in flight than one wave of long ones
+    int64_t x = ((int64_t)num_sms * 48) / ((int64_t)b.n * b.n_layers);
     const int64_t need = (pieces + (int64_t)kThreads * kUnroll - 1) / ((int64_t)kThreads * kUnroll);
     if (x > need) x = need;
     if (x < 1) x = 1;
