@@ -517,6 +517,103 @@ def layer_subset(name: str, layers: int):
     return sub
 
 
+def time_next_rows(f, c, spec, keep, stream, dev, hbm_peak, reps=10):
+    """The rows built beyond the score -> select -> compact path, each timed on the headline's
+    inputs with CUDA events on the launching stream around a CUDA graph of `reps` calls (two
+    untimed calls and one untimed replay first): the p = infinity
+    and query-self-key variants of the whole step, the continuous-row and token-ID messages of
+    the selected positions (hidden-state rows of the model's width), the compaction with the RoPE
+    re-index, and a three-hop chain under the relative chain budget."""
+    import torch
+    import paper_2609_32046_gb300 as cb
+    sh = spec.shape
+    g = torch.Generator(device="cpu").manual_seed(1234)
+
+    def timed(fn):
+        # `reps` calls captured as one CUDA graph and replayed, so the host's enqueue time (the
+        # Python binding) does not show in the device time of these short calls
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize(dev)
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream):
+            for _ in range(reps):
+                fn()
+        gr.replay()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            gr.replay()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / reps
+
+    T = sum(f.Ts)
+    out = {}
+    # p = infinity (App. D.2): the same step with maxima in place of the sums of powers
+    cinf = cb.CacheBack(sh.n_layers, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, spec.m, max(spec.T), len(f.Ks),
+                        p=float("inf"))
+    finf = cb.Filter(cinf, list(zip(f.Ks, f.Vs)), f.Qs, keep, device=dev)
+    ms = timed(lambda: finf.run(stream))
+    cinf.sync_status(stream)
+    out["p_infinity"] = {"ms_per_step": ms, "value": T / (ms / 1e3), "unit": UNIT}
+    del finf, cinf
+    # the query tokens' own keys join the softmax causally (one key per query token and KV head)
+    kq = [(torch.randn((sh.n_layers, q.shape[1], sh.n_kv_heads, sh.head_dim), generator=g) * 0.5)
+          .to(torch.bfloat16).to(dev) for q in f.Qs]
+    fsk = cb.Filter(c, list(zip(f.Ks, f.Vs)), f.Qs, keep, device=dev, query_keys=kq)
+    ms = timed(lambda: fsk.run(stream))
+    c.sync_status(stream)
+    out["query_self_keys"] = {"ms_per_step": ms, "value": T / (ms / 1e3), "unit": UNIT,
+                              "score_kernels": {2: "tcgen05", 1: "mma.sync"}.get(c.score_path(), "none")}
+    del fsk, kq
+    f.run(stream)
+    # messages: hidden-state rows (the model's width, 2 bytes an element) of the selected positions
+    hidden = sh.n_q_heads * sh.head_dim
+    tables = [(torch.randn((Ti, hidden), generator=g)).to(torch.bfloat16).to(dev) for Ti in f.Ts]
+    ids = [torch.randint(0, 151936, (Ti,), generator=g, dtype=torch.int32).to(dev) for Ti in f.Ts]
+    rows = sum(f.budgets)
+    ms = timed(lambda: f.message_rows(tables, stream))
+    b_rows = 2 * rows * hidden * 2
+    out["message_rows"] = {"ms": ms, "bound": "hbm", "bytes": b_rows, "gbs": b_rows / (ms / 1e3) / 1e9,
+                           "frac": b_rows / (ms / 1e3) / 1e9 / hbm_peak, "row_bytes": hidden * 2}
+    ms = timed(lambda: f.message_token_ids(ids, tables, stream))
+    lat = sum(min(Ti, c.cfg.n_latent) for Ti in f.Ts)
+    b_ids = 2 * ((rows - lat) * 4 + lat * hidden * 2)
+    out["message_token_ids"] = {"ms": ms, "bound": "hbm", "bytes": b_ids, "gbs": b_ids / (ms / 1e3) / 1e9}
+    del tables, ids
+    # compaction with K moved to receiver positions (RoPE re-index, App. C.3)
+    rope = dict(base=1.0e6, style=0, pos0=4096)
+    ms = timed(lambda: f.compact(stream, rope=rope))
+    b_c = 2 * 2 * rows * sh.n_layers * sh.n_kv_heads * sh.head_dim * 2
+    out["compact_rope"] = {"ms": ms, "bound": "hbm", "bytes": b_c, "gbs": b_c / (ms / 1e3) / 1e9,
+                           "frac": b_c / (ms / 1e3) / 1e9 / hbm_peak}
+    # chain budgets (App. C.2): three hops of T / 3 new positions each, relative budget
+    T0 = f.Ts[0]
+    T_new = T0 // 3
+    cap = 3 * T_new                        # the longest hop holds T_new + its inherited message
+    cc = cb.CacheBack(sh.n_layers, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, spec.m, cap, 1)
+    K0, V0, Q0 = f.Ks[0], f.Vs[0], f.Qs[0]
+    hops = [(K0[:, :, i * T_new:(i + 1) * T_new].contiguous(), V0[:, :, i * T_new:(i + 1) * T_new].contiguous())
+            for i in range(3)]
+    ch = cb.Chain(cc, cap, keep=keep, mode="relative", device=dev)
+
+    def chain():
+        ch.cur, ch.T_old = 0, 0            # a fresh chain over the same buffers
+        with torch.cuda.stream(stream):
+            for k, v in hops:
+                ch.hop(Q0, k, v, stream=stream)
+    ms = timed(chain)
+    cc.sync_status(stream)
+    out["chain_3_hops"] = {"ms": ms, "value": 3 * T_new / (ms / 1e3), "unit": UNIT,
+                           "note": "new positions scored per second over three hops (each hop also scores "
+                                   "the inherited message); includes copying each hop's new K/V into the chain"}
+    del ch, cc, hops
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args):
     import torch
     import paper_2609_32046_gb300 as cb
@@ -815,6 +912,8 @@ def run_ours(args):
         out["e2e"] = e2e
     if pipelined:
         out["pipelined"] = pipelined
+    if not args.no_next_rows and not args.paged and args.workload == "qwen8b":
+        out["next_rows"] = time_next_rows(f, c, spec, keep, stream, dev, hbm_peak)
     extra = [x for x in (args.workloads or "").split(",") if x]
     if extra and not args.paged:
         del f, c, w, senders, queries, states, states_all, inputs
@@ -846,6 +945,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-pipelined", action="store_true", help="skip the two-steps-in-flight measurement")
     ap.add_argument("--no-graph", action="store_true", help="launch the timed steps directly, not as a CUDA graph")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip timing the rows beyond score/select/compact (p = infinity, self keys, messages, "
+                         "RoPE re-index, chain)")
     ap.add_argument("--cpu-layers", type=int, default=0, help="oracle layers per sample (0: by workload size)")
     ap.add_argument("--paged", type=int, default=0,
                     help="hold each sender cache in pages of this many positions (random page order)")

@@ -143,9 +143,10 @@ cudaError_t launch_compact_rope(const CompactBatch& b, double base, int style, i
         rb->turns[k] = (uint64_t)ldexpl(f, 64);
     }
     const int segs = 2 * b.n_layers * b.n_kv_heads;
-    // about 8 resident blocks per SM over the batch; each block walks a slice of its segment's rows
+    // about 48 blocks per SM over the batch (six waves of eight resident blocks); each block walks a
+    // slice of its segment's rows
     const int rows_per_pass = kThreads / (b.head_dim / 8);
-    int64_t slices = ((int64_t)num_sms * 8 + (int64_t)segs * b.n - 1) / ((int64_t)segs * b.n);
+    int64_t slices = ((int64_t)num_sms * 48) / ((int64_t)segs * b.n);
     const int64_t need = (max_B + rows_per_pass - 1) / rows_per_pass;
     if (slices > need) slices = need;
     if (slices < 1) slices = 1;

@@ -257,8 +257,76 @@ __global__ void __launch_bounds__(kThreads, 2) k_stats(const __grid_constant__ S
 // loaded before any is merged (the partials mostly come from DRAM).
 constexpr int kCombThreads = 256;
 constexpr int kCombBatch = 32;     // slots of a row loaded before they are merged
-template <int TPR>
+constexpr int kSelfChunk = 64;     // query self keys staged in shared memory at a time
+
+// One logit x (log2 domain) into the running offset M and sum L.
+__device__ __forceinline__ void merge_logit1(float x, float& M, float& L) {
+    if (x > M) {
+        L = (M == -INFINITY ? 0.f : L * ex2(M - x)) + 1.f;
+        M = x;
+    } else {
+        L += ex2(x - M);
+    }
+}
+
+// The query tokens' own keys of one block's group (l, g) join its rows' statistics: row (token
+// r, head h) attends to keys 0..r, key u merged on chain u mod 4 in increasing u (NC = 4: the
+// thread merges every chain; NC = 1: only chain c0l).  The block stages the keys in shared memory
+// 64 at a time and each thread holds its query row in registers; the dot products add in the
+// order of the per-row version.  Every thread of the block calls it (it synchronises the block);
+// `act` selects the threads with a row.
+template <int D, int NC>
+__device__ __forceinline__ void self_keys_staged(const ScoreSender& sd, int l, int g, int r_tok, int c0l,
+                                                 const uint16_t* qrow, float sl2e, bool act, float (&M)[NC],
+                                                 float (&L)[NC], uint4* ks) {
+    constexpr int P = D / 8;   // 16-byte pieces of a key
+    uint32_t qw[D / 2];
+#pragma unroll
+    for (int p = 0; p < P; ++p) {
+        const uint4 a = act ? *reinterpret_cast<const uint4*>(qrow + 8 * p) : make_uint4(0u, 0u, 0u, 0u);
+        qw[4 * p] = a.x;
+        qw[4 * p + 1] = a.y;
+        qw[4 * p + 2] = a.z;
+        qw[4 * p + 3] = a.w;
+    }
+    const uint16_t* kbase = sd.kself + (int64_t)l * sd.kss_l + (int64_t)g * sd.kss_h;
+    for (int u0 = 0; u0 < sd.m; u0 += kSelfChunk) {
+        const int nk = sd.m - u0 < kSelfChunk ? sd.m - u0 : kSelfChunk;
+        __syncthreads();   // the previous chunk is no longer read
+        for (int e = threadIdx.x; e < nk * P; e += blockDim.x)
+            ks[e] = *reinterpret_cast<const uint4*>(kbase + (int64_t)(u0 + e / P) * sd.kss_t + 8 * (e % P));
+        __syncthreads();
+        const int uend = r_tok + 1 < u0 + nk ? r_tok + 1 : u0 + nk;
+        if (!act) continue;
+        for (int ub = u0; ub < uend; ub += 4) {
+#pragma unroll
+            for (int k = 0; k < NC; ++k) {
+                const int u = ub + (NC == 1 ? c0l : k);
+                if (u >= uend) break;
+                const uint4* kr = ks + (u - u0) * P;
+                float dot = 0.f;
+#pragma unroll
+                for (int p = 0; p < P; ++p) {
+                    const uint4 b = kr[p];
+                    const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        dot = fmaf(__uint_as_float(qw[4 * p + w] << 16), __uint_as_float(bw[w] << 16), dot);
+                        dot = fmaf(__uint_as_float(qw[4 * p + w] & 0xFFFF0000u), __uint_as_float(bw[w] & 0xFFFF0000u),
+                                   dot);
+                    }
+                }
+                merge_logit1(dot * sl2e, M[k], L[k]);
+            }
+        }
+    }
+}
+
+// SELF: some sender of the batch has query self keys (an instantiation of its own: the staged
+// self keys and the query row in registers would halve the occupancy of the plain merge).
+template <int TPR, bool SELF>
 __global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant__ ScoreBatch bt, int G) {
+    __shared__ uint4 ks_sm[SELF ? kSelfChunk * 16 : 1];   // staged query self keys (d <= 128)
     constexpr int RPB = kCombThreads / TPR;   // rows per block
     constexpr int NC = 4 / TPR;               // chains a thread merges
     const int nS = bt.n_layers * bt.n_kv_heads;
@@ -280,7 +348,7 @@ __global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant_
     const int s = (int)(blk / nrb);
     const int row = (int)(blk % nrb) * RPB + (int)threadIdx.x / TPR;
     const int c0l = TPR == 1 ? 0 : (int)threadIdx.x % TPR;   // the thread's first chain
-    if (row >= rows) return;                                   // (the four threads of a row together)
+    const bool in_rows = row < rows;   // (the four threads of a row together)
     const unsigned gmask = TPR == 1 ? 0u : 0xFu << ((threadIdx.x & 31) & ~3u);
     const int l = s / bt.n_kv_heads, g = s % bt.n_kv_heads;
     const int r_tok = row / G, hh = row - r_tok * G;
@@ -319,10 +387,10 @@ __global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant_
                                 bt.scale_log2e, M[k], L[k]);
     };
     float off = 0.f;
-    if (row < R) {
-        float M[NC], L[NC];
+    float M[NC], L[NC];
 #pragma unroll
-        for (int k = 0; k < NC; ++k) { M[k] = -INFINITY; L[k] = 0.f; }
+    for (int k = 0; k < NC; ++k) { M[k] = -INFINITY; L[k] = 0.f; }
+    if (row < R) {
         const float2* st = bt.stats + sd.stats_off + (int64_t)s * sd.n_chunk1 * R + row;
         for (int cb = 0; cb < sd.n_chunk1; cb += kCombBatch) {
             constexpr int NL = kCombBatch / TPR;   // this thread's slots of the batch
@@ -345,7 +413,14 @@ __global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant_
                 }
             }
         }
-        if (sd.kself) merge_self_keys(M, L);
+    }
+    if (SELF && sd.kself) {   // the whole block (a block's rows belong to one group)
+        if (bt.head_dim == 128)
+            self_keys_staged<128, NC>(sd, l, g, r_tok, c0l, qrow, bt.scale_log2e, row < R, M, L, ks_sm);
+        else
+            self_keys_staged<64, NC>(sd, l, g, r_tok, c0l, qrow, bt.scale_log2e, row < R, M, L, ks_sm);
+    }
+    if (row < R) {
         // A chunk partial whose sum left fp32 range makes the row's sum infinite (pass 1 of the
         // tensor-memory path offsets each chunk by the maximum of its first 32 logits, so a logit
         // far larger later in the chunk overflows exp2).  Such rows, rare, are recomputed here
@@ -392,7 +467,7 @@ __global__ void __launch_bounds__(kCombThreads) k_combine(const __grid_constant_
         off = Mx + log2f(Lx) + log2f((float)G);
         if (c0l == 0) bt.offs[sd.offs_off + (int64_t)s * R + row] = off;
     }
-    if (c0l != 0) return;
+    if (!in_rows || c0l != 0) return;
     if (bt.ext) {
         // the tcgen05 pass 2 adds -off / scale_log2e to the logit inside the contraction
         // (one more K-step against a column of ones): three bf16 terms carry it to ~24 bits
@@ -691,6 +766,8 @@ int64_t combine_rows(const ScoreBatch& b) {
 
 template <int TPR>
 cudaError_t launch_combine_t(const ScoreBatch& b, cudaStream_t st) {
+    bool self = false;
+    for (int i = 0; i < b.n; ++i) self = self || b.s[i].kself != nullptr;
     const int G = b.n_q_heads / b.n_kv_heads;
     const int64_t nS = (int64_t)b.n_layers * b.n_kv_heads;
     constexpr int RPB = kCombThreads / TPR;
@@ -700,7 +777,10 @@ cudaError_t launch_combine_t(const ScoreBatch& b, cudaStream_t st) {
         const int64_t rows = b.ext ? rows_pad128(R) : R;
         nb += nS * ((rows + RPB - 1) / RPB);
     }
-    k_combine<TPR><<<(unsigned)nb, kCombThreads, 0, st>>>(b, G);
+    if (self)
+        k_combine<TPR, true><<<(unsigned)nb, kCombThreads, 0, st>>>(b, G);
+    else
+        k_combine<TPR, false><<<(unsigned)nb, kCombThreads, 0, st>>>(b, G);
     return cudaGetLastError();
 }
 
