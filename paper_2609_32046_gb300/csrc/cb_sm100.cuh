@@ -63,21 +63,9 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint64_t* bar, uint32_t parit
     return ok != 0;
 }
 
-// Wait for phase `parity` of `bar` to complete; gives up after `limit` polls
-// (each poll itself blocks for a hardware-bounded time).  Returns false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit) {
-    for (uint32_t i = 0; i < limit; ++i)
-        if (mbar_try_wait(bar, parity)) return true;
-    return false;
-}
-
 // ---------------------------------------------------------------------------
 // TMA (tiled tensor loads into shared memory, completion on an mbarrier)
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* m) {
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
-}
-
 __device__ __forceinline__ void tma_load_2d(void* smem, const CUtensorMap* m, uint64_t* bar, int32_t x, int32_t y) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
@@ -102,14 +90,6 @@ __device__ __forceinline__ void tma_load_4d(void* smem, const CUtensorMap* m, ui
             smem_u32(smem)),
         "l"(reinterpret_cast<uint64_t>(m)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z), "r"(w)
         : "memory");
-}
-
-// Prefetch a tensor tile into L2 (no shared memory, no completion tracking).
-__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* m, int32_t x, int32_t y, int32_t z, int32_t w) {
-    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
-                     reinterpret_cast<uint64_t>(m)),
-                 "r"(x), "r"(y), "r"(z), "r"(w)
-                 : "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -294,21 +274,6 @@ __device__ __forceinline__ float max_tree1(const float (&x)[32]) {
     return fmax3(w0, w1, fmax3(w2, u[9], u[10]));
 }
 
-// Max of two 32-value register arrays by a tree of 3-input max (depth 4).
-__device__ __forceinline__ float max_tree2(const float (&x)[32], const float (&y)[32]) {
-    float u[22];
-#pragma unroll
-    for (int i = 0; i < 10; ++i) u[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
-    u[10] = fmax3(x[30], x[31], y[0]);
-#pragma unroll
-    for (int i = 0; i < 10; ++i) u[11 + i] = fmax3(y[3 * i + 1], y[3 * i + 2], y[3 * i + 3]);
-    u[21] = y[31];
-    const float w0 = fmax3(u[0], u[1], u[2]), w1 = fmax3(u[3], u[4], u[5]), w2 = fmax3(u[6], u[7], u[8]);
-    const float w3 = fmax3(u[9], u[10], u[11]), w4 = fmax3(u[12], u[13], u[14]), w5 = fmax3(u[15], u[16], u[17]);
-    const float w6 = fmax3(u[18], u[19], u[20]);
-    return fmax3(fmax3(w0, w1, w2), fmax3(w3, w4, w5), fmaxf(w6, u[21]));
-}
-
 __device__ __forceinline__ bool elect_one() {
     uint32_t pred;
     asm volatile(
@@ -317,25 +282,6 @@ __device__ __forceinline__ bool elect_one() {
         "selp.b32 %0, 1, 0, p;\n\t}"
         : "=r"(pred));
     return pred != 0;
-}
-
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
-
-// Named barrier that also returns the AND of `v` over the participating threads,
-// so a group takes one decision (e.g. to abort) without diverging.
-__device__ __forceinline__ bool named_bar_and(int id, int nthreads, bool v) {
-    uint32_t r;
-    asm volatile(
-        "{\n\t.reg .pred p, q;\n\t"
-        "setp.ne.u32 p, %1, 0;\n\t"
-        "bar.red.and.pred q, %2, %3, p;\n\t"
-        "selp.u32 %0, 1, 0, q;\n\t}"
-        : "=r"(r)
-        : "r"((uint32_t)v), "r"(id), "r"(nthreads)
-        : "memory");
-    return r != 0;
 }
 
 }  // namespace sm100
