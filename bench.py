@@ -600,7 +600,7 @@ def time_next_rows(f, c, spec, keep, stream, dev, hbm_peak, reps=10):
     ch = cb.Chain(cc, cap, keep=keep, mode="relative", device=dev)
 
     def chain():
-        ch.cur, ch.T_old = 0, 0            # a fresh chain over the same buffers
+        ch.reset()                         # a fresh chain over the same buffers
         with torch.cuda.stream(stream):
             for k, v in hops:
                 ch.hop(Q0, k, v, stream=stream)

@@ -186,6 +186,11 @@ class Chain:
         self.cur = 0
         self.T_old = 0
 
+    def reset(self):
+        """Start a new chain over the same buffers (the next hop inherits no message)."""
+        self.cur = 0
+        self.T_old = 0
+
     def new_slot(self, T_new: int):
         """Views of the current buffer where the hop's T_new new positions go (after the message)."""
         a, b = self.T_old, self.T_old + int(T_new)
