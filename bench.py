@@ -520,8 +520,8 @@ def layer_subset(name: str, layers: int):
 def time_next_rows(f, c, spec, keep, stream, dev, hbm_peak, reps=10):
     """The rows built beyond the score -> select -> compact path, each timed on the headline's
     inputs with CUDA events on the launching stream around a CUDA graph of `reps` calls (two
-    untimed calls and one untimed replay first): the p = infinity
-    and query-self-key variants of the whole step, the continuous-row and token-ID messages of
+    untimed calls and one untimed replay first): the p = infinity, alpha = 0, per-position and
+    query-self-key variants of the whole step, the continuous-row and token-ID messages of
     the selected positions (hidden-state rows of the model's width), the compaction with the RoPE
     re-index, and a three-hop chain under the relative chain budget."""
     import torch
@@ -559,6 +559,16 @@ def time_next_rows(f, c, spec, keep, stream, dev, hbm_peak, reps=10):
     cinf.sync_status(stream)
     out["p_infinity"] = {"ms_per_step": ms, "value": T / (ms / 1e3), "unit": UNIT}
     del finf, cinf
+    # the selector switches: alpha = 0 (mean query attention, SnapKV-style) and per-position
+    # ranking (span width 1)
+    for name, kw in (("alpha_0", dict(alpha=0.0)), ("per_position_spans", dict(span_width=1))):
+        cs = cb.CacheBack(sh.n_layers, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, spec.m, max(spec.T), len(f.Ks),
+                          **kw)
+        fs = cb.Filter(cs, list(zip(f.Ks, f.Vs)), f.Qs, keep, device=dev)
+        ms = timed(lambda: fs.run(stream))
+        cs.sync_status(stream)
+        out[name] = {"ms_per_step": ms, "value": T / (ms / 1e3), "unit": UNIT}
+        del fs, cs
     # the query tokens' own keys join the softmax causally (one key per query token and KV head)
     kq = [(torch.randn((sh.n_layers, q.shape[1], sh.n_kv_heads, sh.head_dim), generator=g) * 0.5)
           .to(torch.bfloat16).to(dev) for q in f.Qs]
