@@ -422,19 +422,35 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
         const int32_t nsp32 = (int32_t)nsp;
         const unsigned below = (1u << lane) - 1u;
         int32_t* const idx = sd.idx;
-        for (int32_t j = warp; j < nsp32; j += kWarps) {
-            const int32_t lo = j * w, hi = lo + w < T32 ? lo + w : T32;
-            const int32_t run = span_run[j];
-            const int32_t left = lo + (run & 0xffff) - 1, right = lo + (run >> 16) - 1;
-            if (right < left && lo >= fa && hi <= fb) continue;   // nothing of this span is kept
-            int32_t base = span_at[j];
-            for (int32_t c0 = lo; c0 < hi; c0 += 32) {
-                const int32_t t = c0 + lane;
-                const bool sel = t < hi && (t < fa || t >= fb || (t >= left && t <= right));
-                const unsigned m = __ballot_sync(0xffffffffu, sel);
-                const int32_t o = base + __popc(m & below);
-                if (sel && o < B32) idx[o] = t;
-                base += __popc(m);
+        // each warp takes 32 spans at a time: one lane a span finds whether anything of it is
+        // kept, and the warp then writes only those spans
+        for (int32_t jb = warp * 32; jb < nsp32; jb += kWarps * 32) {
+            const int32_t jl = jb + lane;
+            int32_t run = 0;
+            bool kept = false;
+            if (jl < nsp32) {
+                const int32_t lo = jl * w, hi = lo + w < T32 ? lo + w : T32;
+                run = span_run[jl];
+                const int32_t left = lo + (run & 0xffff) - 1, right = lo + (run >> 16) - 1;
+                kept = !(right < left && lo >= fa && hi <= fb);
+            }
+            unsigned km = __ballot_sync(0xffffffffu, kept);
+            while (km) {
+                const int src = __ffs(km) - 1;
+                km &= km - 1;
+                const int32_t j = jb + src;
+                const int32_t rj = __shfl_sync(0xffffffffu, run, src);
+                const int32_t lo = j * w, hi = lo + w < T32 ? lo + w : T32;
+                const int32_t left = lo + (rj & 0xffff) - 1, right = lo + (rj >> 16) - 1;
+                int32_t base = span_at[j];
+                for (int32_t c0 = lo; c0 < hi; c0 += 32) {
+                    const int32_t t = c0 + lane;
+                    const bool sel = t < hi && (t < fa || t >= fb || (t >= left && t <= right));
+                    const unsigned m = __ballot_sync(0xffffffffu, sel);
+                    const int32_t o = base + __popc(m & below);
+                    if (sel && o < B32) idx[o] = t;
+                    base += __popc(m);
+                }
             }
         }
     }
