@@ -51,6 +51,8 @@ CASES = [
     ("self_keys_g4", (2, 32, 8, 128), [700], 40, 0.25, dict(self_keys=True)),
     ("self_keys_g2_d64", (2, 8, 4, 64), [333], 17, 0.3, dict(self_keys=True)),
     ("self_keys_fan_in_m128", (1, 16, 4, 128), [300, 129], 128, 0.25, dict(self_keys=True)),
+    # 100 query tokens: the staged self keys come in a chunk of 64 and one of 36
+    ("self_keys_m100_two_chunks", (2, 8, 2, 128), [500], 100, 0.3, dict(self_keys=True)),
     # more senders than one tcgen05 launch takes (32): two launches per pass
     ("forty_senders", (1, 8, 2, 128), [97 + 13 * i for i in range(40)], 8, 0.3, {}),
 ]
